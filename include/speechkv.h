@@ -1,0 +1,210 @@
+/*
+ * speechkv.h -- C ABI of the GB300 (sm_103a) SpeechKV decode hot path.
+ *
+ * SpeechKV ("Compress the Cache, Not the Speech Embedding", Sec. III-B)
+ * compresses the speech span of a speech LLM's KV cache: from layer l0 on,
+ * every window of w consecutive speech frames is replaced by one pooled key
+ * and one pooled value, weighted by a softmax over a learned linear gate of
+ * the keys (Eq. (pool)); text positions are kept.  Each decode step then
+ * appends the new token's key/value and runs grouped-query attention of the
+ * full-resolution query over the shorter cache (Eq. (attn)).  The pooling
+ * runs once at prefill and its result is what the cache stores (Sec. III-C).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Pointers marked "dev" are CUDA device pointers; the caller owns every
+ *   buffer, including the decode workspace.  Nothing here allocates device
+ *   memory per call.
+ * - Calls are asynchronous and ordered on `stream`; none synchronises the
+ *   host.  Argument errors are detected on the host before any launch and
+ *   returned as a status; nothing is launched then.
+ * - Errors that depend on device-resident values (a cache that is full, a
+ *   length beyond its capacity, inconsistent lengths, a bounded wait that
+ *   ran out) set a per-device error word instead of faulting; the offending
+ *   write is skipped.  speechkv_check_device_error() reads and clears it.
+ * - Element types: SPEECHKV_F32 or SPEECHKV_BF16 storage for keys, values,
+ *   queries and outputs; all arithmetic is fp32.  Head dim d is 64 or 128.
+ * - Data pointers (keys, values, queries, outputs, caches, workspace) must be
+ *   16-byte aligned.
+ * - Layers are counted from 0; layer `layer` is pooled iff layer >= l0, so
+ *   the paper's default "l0 = 5, first 4 layers full resolution" is l0 = 4.
+ *
+ * Cache layout (one buffer per layer for K and one for V)
+ * -------------------------------------------------------
+ * Request b owns rows [cache_off[b], cache_off[b+1]) of capacity
+ * cap_b = cache_off[b+1] - cache_off[b].  Its block is head-major:
+ * element (b, h, t, c) lives at ((cache_off[b] * H_kv + h * cap_b + t) * d + c)
+ * for KV head h, cached row t < cap_b, channel c.  One (request, head) is thus
+ * a single contiguous run of rows, which the decode kernel streams with bulk
+ * asynchronous copies.  Rows are, in order: the P text tokens before the
+ * speech, the n = ceil(T / w_eff) pooled speech entries, the N text tokens
+ * after the speech, then the generated tokens.  len[b] (int32, dev) counts the
+ * rows in use.
+ */
+#ifndef SPEECHKV_H_
+#define SPEECHKV_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SPEECHKV_OK = 0,
+    SPEECHKV_ERR_INVALID_ARG = 1,  /* bad pointer, size, shape or length   */
+    SPEECHKV_ERR_UNSUPPORTED = 2,  /* valid but not built (d, group, dtype) */
+    SPEECHKV_ERR_CUDA = 3,         /* a CUDA runtime call failed            */
+    SPEECHKV_ERR_CAPACITY = 4,     /* a cache row would pass its capacity   */
+    SPEECHKV_ERR_TIMEOUT = 5,      /* a bounded device wait ran out         */
+    SPEECHKV_ERR_WORKSPACE = 6     /* decode workspace too small            */
+} speechkv_status;
+
+typedef enum { SPEECHKV_F32 = 0, SPEECHKV_BF16 = 1 } speechkv_dtype;
+
+/* Largest batch speechkv_decode_attn accepts (its per-CTA length table). */
+#define SPEECHKV_MAX_BATCH 2048
+
+/* Human-readable name of a status (static string, never NULL). */
+const char *speechkv_status_string(speechkv_status status);
+
+/*
+ * Cached rows of one request at one layer (Sec. III-B: speech pooled in
+ * windows of w from layer l0 on, text unchanged):
+ *   P + ceil(T / w_eff) + N + G,  w_eff = (layer >= l0 ? w : 1).
+ * P / N: text tokens before / after the speech, T: speech frames, G: tokens
+ * generated so far.  A partial last window still yields one entry.  Pure host
+ * function; returns -1 for negative counts, w < 1, layer < 0 or l0 < 0.
+ */
+int64_t speechkv_compressed_len(int32_t P, int32_t T, int32_t N, int32_t G,
+                                int32_t w, int32_t layer, int32_t l0);
+
+/*
+ * speechkv_pool -- Eq. (pool), run once per request and layer at prefill.
+ *
+ * For every request b and KV head h, writes the cache rows described above
+ * from the full-resolution prefill keys/values:
+ *   - text rows are copied bit-exactly;
+ *   - speech window i (frames i*w_eff .. min((i+1)*w_eff, T) - 1 of the
+ *     speech span) becomes one row: logits z_j = gate[h] . k_j, weights
+ *     alpha = softmax(z) over the window, k^ = sum alpha_j k_j and
+ *     v^ = sum alpha_j v_j (values use the keys' weights), rounded once to the
+ *     storage type (round to nearest even);
+ *   - when layer < l0 (w_eff = 1) every row is copied bit-exactly.
+ * Then sets len[b] = P[b] + ceil(T[b] / w_eff) + N[b].
+ *
+ * k_full, v_full  dev, [full_rows][H_kv][d] token-major prefill keys/values;
+ *                 request b's rows are [full_off[b], full_off[b+1]), which
+ *                 must hold exactly P[b] + T[b] + N[b] rows.
+ * full_off        dev int64 [B+1], non-decreasing, full_off[B] <= full_rows.
+ * P, T, N         dev int32 [B]: text before, speech frames, text after.
+ * gate            dev fp32 [H_kv][d]: the gate vector u of g(k) = u . k for
+ *                 this layer, one per KV head (no bias: a bias is constant
+ *                 over a window and cancels in the softmax).
+ * k_cache,v_cache dev, this layer's cache blocks (layout above).
+ * cache_off       dev int64 [B+1], capacities in rows.
+ * len             dev int32 [B], written.
+ * full_rows       host: rows in k_full / v_full (sizes the launch).
+ * w               window (>= 1); layer, l0 as above.
+ * Errors: host-checked arguments return a status.  On the device, a request
+ * whose rows do not match P+T+N sets SPEECHKV_ERR_INVALID_ARG; a request
+ * whose pooled rows exceed its capacity sets SPEECHKV_ERR_CAPACITY (rows
+ * beyond the capacity are not written and len is clamped to it).
+ */
+speechkv_status speechkv_pool(const void *k_full, const void *v_full,
+                              const int64_t *full_off, const int32_t *P,
+                              const int32_t *T, const int32_t *N,
+                              const float *gate, void *k_cache, void *v_cache,
+                              const int64_t *cache_off, int32_t *len,
+                              int32_t B, int64_t full_rows, int32_t H_kv,
+                              int32_t d, int32_t w, int32_t layer, int32_t l0,
+                              speechkv_dtype dtype, cudaStream_t stream);
+
+/*
+ * speechkv_append -- one decode step's cache update (Sec. III-C: decoding
+ * appends each new token to the cache uncompressed).
+ *
+ * For every request b: writes k_new[b], v_new[b] ([H_kv][d]) as cached row
+ * len[b] of request b, then len[b] += 1.  A request whose cache is full
+ * (len[b] >= cap_b, or len[b] < 0) is left untouched and sets
+ * SPEECHKV_ERR_CAPACITY in the device error word.
+ *
+ * k_new, v_new   dev, [B][H_kv][d].
+ * k_cache, v_cache, cache_off, len: as for speechkv_pool (len read+written).
+ * w, layer, l0   validated only (w >= 1, layer >= 0, l0 >= 0).
+ */
+speechkv_status speechkv_append(const void *k_new, const void *v_new,
+                                void *k_cache, void *v_cache,
+                                const int64_t *cache_off, int32_t *len,
+                                int32_t B, int32_t H_kv, int32_t d, int32_t w,
+                                int32_t layer, int32_t l0,
+                                speechkv_dtype dtype, cudaStream_t stream);
+
+/*
+ * Bytes of workspace speechkv_decode_attn needs for a batch of B requests
+ * with the given heads and head dim, launched on `grid_ctas` CTAs (0 = the
+ * automatic grid, sized from the current device's SM count).  The workspace
+ * holds split-K partial results and one arrival counter per (request, KV
+ * head).  Returns 0 for invalid arguments.
+ */
+size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv,
+                                      int32_t d, int32_t grid_ctas);
+
+/*
+ * speechkv_decode_attn -- Eq. (attn) for one decode step at one layer.
+ *
+ * For every request b and query head hq (KV head h = hq / (H_q / H_kv)):
+ *   s_j = scale * q[b][hq] . k_j  for the cached rows j < len[b],
+ *   out[b][hq] = sum_j softmax(s)_j v_j,
+ * rounded once to the storage type.  scale <= 0 selects 1 / sqrt(d).  A
+ * request with len[b] == 0 gets a zero output.  len[b] > cap_b sets
+ * SPEECHKV_ERR_CAPACITY and attends over cap_b rows.
+ *
+ * The work (every request's rows times its KV heads) is cut evenly over a
+ * persistent grid; every CTA streams its share from HBM once, serving all
+ * H_q / H_kv query heads of a KV head from one read, and pieces of a
+ * (request, head) processed by several CTAs are merged with a log-sum-exp
+ * combine by the CTA that finishes last (no CTA ever waits for another).
+ *
+ * q            dev, [B][H_q][d].
+ * k_cache, v_cache, cache_off, len: as for speechkv_pool (len read only).
+ * out          dev, [B][H_q][d], written.
+ * H_q / H_kv   must be 1, 2 or 4; d must be 64 or 128; B <= SPEECHKV_MAX_BATCH.
+ * w, layer, l0 validated only.
+ * grid_ctas    CTAs to launch; 0 = automatic (one per SM times the
+ *              kernel's residency).  Results do not depend on it beyond
+ *              floating-point summation order.
+ * workspace    dev, >= speechkv_decode_workspace_size(B, H_q, H_kv, d,
+ *              grid_ctas) bytes.  It must be zero-filled once before its
+ *              first use; every call leaves its counters at zero again.
+ *              Calls that run concurrently need separate workspaces.  After
+ *              a device error, zero it again.
+ */
+speechkv_status speechkv_decode_attn(const void *q, const void *k_cache,
+                                     const void *v_cache,
+                                     const int64_t *cache_off,
+                                     const int32_t *len, void *out,
+                                     float scale, int32_t B, int32_t H_q,
+                                     int32_t H_kv, int32_t d, int32_t w,
+                                     int32_t layer, int32_t l0,
+                                     int32_t grid_ctas, void *workspace,
+                                     size_t workspace_bytes,
+                                     speechkv_dtype dtype,
+                                     cudaStream_t stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the current device's error
+ * word.  Returns SPEECHKV_OK when no kernel reported an error since the last
+ * check, else the first error reported (CAPACITY, INVALID_ARG or TIMEOUT),
+ * or SPEECHKV_ERR_CUDA if the synchronisation itself failed.
+ */
+speechkv_status speechkv_check_device_error(cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPEECHKV_H_ */

@@ -1,0 +1,280 @@
+// C ABI of libspeechkv: argument checks, per-device state and dispatch to the
+// kernels (pool.cu, append.cu, decode_attn.cu).  Declarations and the full
+// contract of every entry point are in include/speechkv.h.
+#include <math.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "launch.h"
+#include "speechkv.h"
+
+// The per-device error word: kernels record the first device-side error here
+// (atomicCAS from 0); speechkv_check_device_error reads and clears it.  A
+// module-scope variable, so the library allocates nothing for it.
+__device__ int speechkv_error_word;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr int kDecodeKinds = 12;  // dtype x d x group
+
+struct DeviceState {
+    int *err = nullptr;  // device address of speechkv_error_word
+    int num_sms = 0;
+    int decode_ctas_per_sm[kDecodeKinds] = {};
+};
+
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+
+speechkv_status current_device(int *dev_out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return SPEECHKV_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return SPEECHKV_ERR_UNSUPPORTED;
+    *dev_out = dev;
+    return SPEECHKV_OK;
+}
+
+// Per-device set-up on first use: the error word's device address (which is
+// what kernels must be given; the host-side symbol is not a device address)
+// and the SM count.
+speechkv_status device_state(DeviceState **out) {
+    int dev = 0;
+    speechkv_status st = current_device(&dev);
+    if (st != SPEECHKV_OK) return st;
+    std::lock_guard<std::mutex> lock(g_mu);
+    DeviceState &s = g_dev[dev];
+    if (!s.err) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, speechkv_error_word) != cudaSuccess) return SPEECHKV_ERR_CUDA;
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+            sms <= 0)
+            return SPEECHKV_ERR_CUDA;
+        s.num_sms = sms;
+        s.err = static_cast<int *>(p);
+    }
+    *out = &s;
+    return SPEECHKV_OK;
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool valid_dtype(speechkv_dtype dt) { return dt == SPEECHKV_F32 || dt == SPEECHKV_BF16; }
+
+int decode_kind(speechkv_dtype dt, int d, int group) {
+    const int g = group == 1 ? 0 : (group == 2 ? 1 : 2);
+    return (dt == SPEECHKV_BF16 ? 6 : 0) + (d == 128 ? 3 : 0) + g;
+}
+
+// Automatic decode grid: one CTA per SM times the kernel's residency (at most
+// two).  Workspace sizing uses the upper bound kAutoCtasPerSmMax.
+constexpr int kAutoCtasPerSmMax = 2;
+
+speechkv_status decode_auto_grid(DeviceState *s, speechkv_dtype dt, int d, int group,
+                                 int *grid) {
+    const int kind = decode_kind(dt, d, group);
+    int per_sm;
+    {
+        std::lock_guard<std::mutex> lock(g_mu);
+        per_sm = s->decode_ctas_per_sm[kind];
+    }
+    if (per_sm == 0) {
+        per_sm = speechkv::decode_ctas_per_sm(dt, d, group);
+        if (per_sm <= 0) return SPEECHKV_ERR_CUDA;
+        if (per_sm > kAutoCtasPerSmMax) per_sm = kAutoCtasPerSmMax;
+        std::lock_guard<std::mutex> lock(g_mu);
+        s->decode_ctas_per_sm[kind] = per_sm;
+    }
+    *grid = s->num_sms * per_sm;
+    return SPEECHKV_OK;
+}
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Workspace layout: counters [B*H_kv] int32 (256-byte padded), then partial
+// slots [grid + B*H_kv][slot_floats] fp32.
+size_t workspace_bytes(int B, int H_q, int H_kv, int d, int grid) {
+    const size_t S = (size_t)B * H_kv;
+    const size_t slot = (size_t)speechkv::decode_slot_floats(d, H_q / H_kv);
+    return round_up(S * 4, 256) + ((size_t)grid + S) * slot * 4;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *speechkv_status_string(speechkv_status status) {
+    switch (status) {
+        case SPEECHKV_OK: return "ok";
+        case SPEECHKV_ERR_INVALID_ARG: return "invalid argument";
+        case SPEECHKV_ERR_UNSUPPORTED: return "unsupported configuration";
+        case SPEECHKV_ERR_CUDA: return "CUDA runtime error";
+        case SPEECHKV_ERR_CAPACITY: return "cache capacity exceeded";
+        case SPEECHKV_ERR_TIMEOUT: return "bounded device wait timed out";
+        case SPEECHKV_ERR_WORKSPACE: return "workspace too small";
+    }
+    return "unknown status";
+}
+
+int64_t speechkv_compressed_len(int32_t P, int32_t T, int32_t N, int32_t G, int32_t w,
+                                int32_t layer, int32_t l0) {
+    if (P < 0 || T < 0 || N < 0 || G < 0 || w < 1 || layer < 0 || l0 < 0) return -1;
+    const int64_t we = layer >= l0 ? w : 1;
+    return (int64_t)P + ((int64_t)T + we - 1) / we + N + G;
+}
+
+speechkv_status speechkv_pool(const void *k_full, const void *v_full, const int64_t *full_off,
+                              const int32_t *P, const int32_t *T, const int32_t *N,
+                              const float *gate, void *k_cache, void *v_cache,
+                              const int64_t *cache_off, int32_t *len, int32_t B,
+                              int64_t full_rows, int32_t H_kv, int32_t d, int32_t w,
+                              int32_t layer, int32_t l0, speechkv_dtype dtype,
+                              cudaStream_t stream) {
+    if (B < 0 || full_rows < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!full_off || !P || !T || !N || !gate || !k_cache || !v_cache || !cache_off || !len ||
+        (full_rows > 0 && (!k_full || !v_full)))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(k_full, 16) || !aligned(v_full, 16) || !aligned(k_cache, 16) ||
+        !aligned(v_cache, 16) || !aligned(full_off, 8) || !aligned(cache_off, 8) ||
+        !aligned(P, 4) || !aligned(T, 4) || !aligned(N, 4) || !aligned(len, 4) ||
+        !aligned(gate, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::PoolArgs a;
+    a.k_full = k_full;
+    a.v_full = v_full;
+    a.full_off = full_off;
+    a.P = P;
+    a.T = T;
+    a.N = N;
+    a.gate = gate;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.B = B;
+    a.full_rows = full_rows;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.w_eff = layer >= l0 ? w : 1;
+    a.dtype = dtype;
+    a.err = s->err;
+    return speechkv::launch_pool(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                       : SPEECHKV_ERR_CUDA;
+}
+
+speechkv_status speechkv_append(const void *k_new, const void *v_new, void *k_cache,
+                                void *v_cache, const int64_t *cache_off, int32_t *len,
+                                int32_t B, int32_t H_kv, int32_t d, int32_t w, int32_t layer,
+                                int32_t l0, speechkv_dtype dtype, cudaStream_t stream) {
+    if (B < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!k_new || !v_new || !k_cache || !v_cache || !cache_off || !len)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_cache, 16) ||
+        !aligned(v_cache, 16) || !aligned(cache_off, 8) || !aligned(len, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::AppendArgs a;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.B = B;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.dtype = dtype;
+    a.err = s->err;
+    return speechkv::launch_append(a, stream) == cudaSuccess ? SPEECHKV_OK : SPEECHKV_ERR_CUDA;
+}
+
+size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv, int32_t d,
+                                      int32_t grid_ctas) {
+    if (B < 0 || H_kv < 1 || H_q < 1 || H_q % H_kv != 0 || grid_ctas < 0) return 0;
+    if (!speechkv::decode_supported(SPEECHKV_BF16, d, H_q / H_kv)) return 0;
+    int grid = grid_ctas;
+    if (grid == 0) {
+        DeviceState *s = nullptr;
+        if (device_state(&s) != SPEECHKV_OK) return 0;
+        grid = s->num_sms * kAutoCtasPerSmMax;
+    }
+    return workspace_bytes(B, H_q, H_kv, d, grid);
+}
+
+speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const void *v_cache,
+                                     const int64_t *cache_off, const int32_t *len, void *out,
+                                     float scale, int32_t B, int32_t H_q, int32_t H_kv,
+                                     int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                                     speechkv_dtype dtype, cudaStream_t stream) {
+    if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
+        grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!q || !k_cache || !v_cache || !cache_off || !len || !out)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+        !aligned(cache_off, 8) || !aligned(len, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    int grid = grid_ctas;
+    if (grid == 0) {
+        st = decode_auto_grid(s, dtype, d, H_q / H_kv, &grid);
+        if (st != SPEECHKV_OK) return st;
+    }
+    const size_t need = workspace_bytes(B, H_q, H_kv, d, grid);
+    if (!workspace || workspace_bytes_in < need || !aligned(workspace, 16))
+        return SPEECHKV_ERR_WORKSPACE;
+    speechkv::DecodeArgs a;
+    a.q = q;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.out = out;
+    a.scale = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
+    a.B = B;
+    a.H_q = H_q;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.dtype = dtype;
+    a.counters = static_cast<int *>(workspace);
+    a.partials = reinterpret_cast<float *>(static_cast<char *>(workspace) +
+                                           round_up((size_t)B * H_kv * 4, 256));
+    a.err = s->err;
+    return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                   : SPEECHKV_ERR_CUDA;
+}
+
+speechkv_status speechkv_check_device_error(cudaStream_t stream) {
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return SPEECHKV_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, speechkv_error_word, sizeof(int)) != cudaSuccess)
+        return SPEECHKV_ERR_CUDA;
+    const int zero = 0;
+    if (v != 0 && cudaMemcpyToSymbol(speechkv_error_word, &zero, sizeof(int)) != cudaSuccess)
+        return SPEECHKV_ERR_CUDA;
+    return static_cast<speechkv_status>(v);
+}
+
+}  // extern "C"

@@ -1,0 +1,63 @@
+// speechkv_append: one decode step's cache update (Sec. III-C: the cache is
+// compressed once at prefill; every generated token then adds one
+// full-resolution key/value per layer).
+//
+// One CTA per request: all threads read len[b] first, copy the token's
+// [H_kv][d] key and value into row len[b] of every head's run with 16-byte
+// stores, and after a barrier one thread advances len[b].  A full cache is
+// reported through the error word and left untouched.
+#include "common.cuh"
+#include "launch.h"
+
+namespace speechkv {
+namespace {
+
+template <typename T>
+__global__ void __launch_bounds__(256)
+    append_kernel(const T *__restrict__ kn, const T *__restrict__ vn, T *__restrict__ kc,
+                  T *__restrict__ vc, const int64_t *__restrict__ cache_off,
+                  int32_t *__restrict__ len, int H_kv, int D, int *__restrict__ err) {
+    constexpr int kPerVec = 16 / (int)sizeof(T);
+    const int b = blockIdx.x;
+    const int64_t L = len[b];
+    const int64_t base = cache_off[b];
+    const int64_t cap = cache_off[b + 1] - base;
+    if (base < 0 || cap < 0) {
+        if (threadIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
+        return;
+    }
+    if (L < 0 || L >= cap) {
+        if (threadIdx.x == 0) report_error(err, SPEECHKV_ERR_CAPACITY);
+        return;  // uniform: every thread took the same branch
+    }
+    const int nvec = H_kv * D / kPerVec;  // 16-byte vectors per tensor
+    for (int i = threadIdx.x; i < 2 * nvec; i += blockDim.x) {
+        const int tensor = i >= nvec;
+        const int e = (i - tensor * nvec) * kPerVec;  // element within [H_kv][d]
+        const int h = e / D, c = e - h * D;
+        const T *src = (tensor ? vn : kn) + (int64_t)b * H_kv * D + e;
+        T *dst = (tensor ? vc : kc) + (base * H_kv + (int64_t)h * cap + L) * D + c;
+        copy_bytes<16>(dst, src);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) len[b] = (int32_t)(L + 1);
+}
+
+}  // namespace
+
+cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream) {
+    if (a.dtype == SPEECHKV_F32)
+        append_kernel<float><<<a.B, 256, 0, stream>>>(
+            static_cast<const float *>(a.k_new), static_cast<const float *>(a.v_new),
+            static_cast<float *>(a.k_cache), static_cast<float *>(a.v_cache), a.cache_off, a.len,
+            a.H_kv, a.d, a.err);
+    else
+        append_kernel<__nv_bfloat16><<<a.B, 256, 0, stream>>>(
+            static_cast<const __nv_bfloat16 *>(a.k_new),
+            static_cast<const __nv_bfloat16 *>(a.v_new),
+            static_cast<__nv_bfloat16 *>(a.k_cache), static_cast<__nv_bfloat16 *>(a.v_cache),
+            a.cache_off, a.len, a.H_kv, a.d, a.err);
+    return cudaGetLastError();
+}
+
+}  // namespace speechkv

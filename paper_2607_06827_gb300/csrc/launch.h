@@ -1,0 +1,60 @@
+// Host-side launchers of the SpeechKV kernels (internal to libspeechkv).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "speechkv.h"
+
+namespace speechkv {
+
+struct PoolArgs {
+    const void *k_full, *v_full;
+    const int64_t *full_off;
+    const int32_t *P, *T, *N;
+    const float *gate;
+    void *k_cache, *v_cache;
+    const int64_t *cache_off;
+    int32_t *len;
+    int32_t B;
+    int64_t full_rows;
+    int32_t H_kv, d, w_eff;
+    speechkv_dtype dtype;
+    int *err;
+};
+cudaError_t launch_pool(const PoolArgs &a, int num_sms, cudaStream_t stream);
+
+struct AppendArgs {
+    const void *k_new, *v_new;
+    void *k_cache, *v_cache;
+    const int64_t *cache_off;
+    int32_t *len;
+    int32_t B, H_kv, d;
+    speechkv_dtype dtype;
+    int *err;
+};
+cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream);
+
+struct DecodeArgs {
+    const void *q, *k_cache, *v_cache;
+    const int64_t *cache_off;
+    const int32_t *len;
+    void *out;
+    float scale;  // > 0
+    int32_t B, H_q, H_kv, d;
+    speechkv_dtype dtype;
+    float *partials;   // [grid + B*H_kv][slot_floats]
+    int *counters;     // [B*H_kv]
+    int *err;
+};
+
+// Whether (dtype, d, group) has a compiled decode kernel.
+bool decode_supported(speechkv_dtype dtype, int d, int group);
+// Resident CTAs per SM of that kernel on the current device (0 on error).
+int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group);
+// Floats per partial-result slot (m, l and o for every query head of a group).
+int decode_slot_floats(int d, int group);
+cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream);
+
+}  // namespace speechkv

@@ -1,0 +1,159 @@
+"""Python binding of libspeechkv (the C ABI in include/speechkv.h).
+
+Argument marshalling only: tensors are passed as raw device pointers, every
+step runs in the library's CUDA kernels, and there is no CPU fallback -- if
+the library is missing or was built for another machine, loading raises.
+Function names and argument order follow the C entry points.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libspeechkv.so")
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_CAPACITY, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
+F32, BF16 = 0, 1
+MAX_BATCH = 2048
+
+# Every function the header declares: name -> (restype, argtypes)
+_P = ctypes.c_void_p
+_I32, _I64, _F, _SZ = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+SIGNATURES = {
+    "speechkv_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+    "speechkv_compressed_len": (_I64, [_I32] * 7),
+    "speechkv_pool": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
+                                     _I32, _I64, _I32, _I32, _I32, _I32, _I32,
+                                     ctypes.c_int, _P]),
+    "speechkv_append": (ctypes.c_int, [_P, _P, _P, _P, _P, _P,
+                                       _I32, _I32, _I32, _I32, _I32, _I32,
+                                       ctypes.c_int, _P]),
+    "speechkv_decode_workspace_size": (_SZ, [_I32] * 5),
+    "speechkv_decode_attn": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _F,
+                                            _I32, _I32, _I32, _I32, _I32, _I32,
+                                            _I32, _I32, _P, _SZ, ctypes.c_int,
+                                            _P]),
+    "speechkv_check_device_error": (ctypes.c_int, [_P]),
+}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class SpeechKVError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} ({status})")
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libspeechkv.so (built by ``paper_2607_06827_gb300.build``)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(path):
+            raise RuntimeError(
+                f"{path} is missing: build it with paper_2607_06827_gb300.build.build() "
+                "(there is no fallback implementation)")
+        lib = ctypes.CDLL(path)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype, fn.argtypes = res, args
+        _lib = lib
+        return lib
+
+
+def status_string(status: int) -> str:
+    return load().speechkv_status_string(status).decode()
+
+
+def _check(status: int, where: str):
+    if status != OK:
+        raise SpeechKVError(status, where)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _ptr(t: torch.Tensor | None):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def compressed_len(P: int, T: int, N: int, G: int, w: int, layer: int, l0: int) -> int:
+    return load().speechkv_compressed_len(P, T, N, G, w, layer, l0)
+
+
+def pool(k_full, v_full, full_off, P, T, N, gate, k_cache, v_cache, cache_off, length,
+         w: int, layer: int, l0: int, stream=None):
+    """speechkv_pool: k_full/v_full [full_rows, H_kv, d]; full_off/cache_off
+    int64 [B+1]; P/T/N/length int32 [B]; gate fp32 [H_kv, d]."""
+    B = length.numel()
+    full_rows, H_kv, d = k_full.shape
+    _check(load().speechkv_pool(
+        _ptr(k_full), _ptr(v_full), _ptr(full_off), _ptr(P), _ptr(T), _ptr(N),
+        _ptr(gate), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off), _ptr(length),
+        B, full_rows, H_kv, d, w, layer, l0, _dtype_code(k_full), _stream(stream)),
+        "speechkv_pool")
+
+
+def append(k_new, v_new, k_cache, v_cache, cache_off, length, w: int, layer: int, l0: int,
+           stream=None):
+    """speechkv_append: k_new/v_new [B, H_kv, d]; length int32 [B] (in/out)."""
+    B, H_kv, d = k_new.shape
+    _check(load().speechkv_append(
+        _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off),
+        _ptr(length), B, H_kv, d, w, layer, l0, _dtype_code(k_new), _stream(stream)),
+        "speechkv_append")
+
+
+def decode_workspace_size(B: int, H_q: int, H_kv: int, d: int, grid_ctas: int = 0) -> int:
+    n = load().speechkv_decode_workspace_size(B, H_q, H_kv, d, grid_ctas)
+    if n == 0:
+        raise SpeechKVError(ERR_INVALID_ARG, "speechkv_decode_workspace_size")
+    return n
+
+
+def new_workspace(B: int, H_q: int, H_kv: int, d: int, grid_ctas: int = 0,
+                  device=None) -> torch.Tensor:
+    """A zero-filled workspace of the size speechkv_decode_attn needs."""
+    n = decode_workspace_size(B, H_q, H_kv, d, grid_ctas)
+    return torch.zeros((n + 15) // 16 * 16, dtype=torch.uint8, device=device or "cuda")
+
+
+def decode_attn(q, k_cache, v_cache, cache_off, length, out, workspace, w: int, layer: int,
+                l0: int, H_kv: int, scale: float = 0.0, grid_ctas: int = 0, stream=None):
+    """speechkv_decode_attn: q/out [B, H_q, d]; caches in the head-major
+    per-request layout; length int32 [B]."""
+    B, H_q, d = q.shape
+    _check(load().speechkv_decode_attn(
+        _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off), _ptr(length), _ptr(out),
+        float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas, _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _dtype_code(q), _stream(stream)),
+        "speechkv_decode_attn")
+
+
+def check_device_error(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device error status."""
+    return load().speechkv_check_device_error(_stream(stream))

@@ -1,0 +1,88 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every entry point
+include/speechkv.h declares; host-only helpers and host-side argument checks
+work without a GPU (no kernel is launched here)."""
+import os
+import re
+
+import pytest
+
+from paper_2607_06827_gb300 import inputs
+from tests import harness as H
+
+HEADER = os.path.join(H.ROOT, "include", "speechkv.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(speechkv_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_the_path():
+    names = _declared()
+    for n in ("speechkv_pool", "speechkv_append", "speechkv_decode_attn",
+              "speechkv_compressed_len", "speechkv_decode_workspace_size",
+              "speechkv_check_device_error", "speechkv_status_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol():
+    sk = H.lib()
+    lib = sk.load()
+    for name in _declared():
+        assert hasattr(lib, name), name
+        assert name in sk.SIGNATURES, f"binding lacks {name}"
+    assert set(sk.SIGNATURES) == set(_declared())
+
+
+def test_compressed_len_matches_oracle(oracle):
+    sk = H.lib()
+    for wl in (inputs.qwen_ragged(), inputs.tiny_fp32(), inputs.qwen_single(),
+               inputs.qwen_long_audio(20, 8)):
+        for layer in (0, wl.l0 - 1 if wl.l0 > 0 else 0, wl.l0, wl.L - 1):
+            for b in range(wl.B):
+                args = (wl.P[b], wl.T[b], wl.N[b], wl.G[b], wl.w, layer, wl.l0)
+                assert sk.compressed_len(*args) == oracle.compressed_len(*args)
+    for T in range(0, 50):
+        for w in range(1, 9):
+            assert sk.compressed_len(3, T, 2, 1, w, 1, 1) == oracle.compressed_len(3, T, 2, 1, w, 1, 1)
+    assert sk.compressed_len(0, 3, 0, 0, 0, 0, 0) == -1
+    assert sk.compressed_len(0, -3, 0, 0, 4, 0, 0) == -1
+
+
+def test_status_strings():
+    sk = H.lib()
+    assert sk.status_string(sk.OK) == "ok"
+    assert "capacity" in sk.status_string(sk.ERR_CAPACITY)
+    assert sk.status_string(99) == "unknown status"
+
+
+def test_host_argument_checks_without_gpu():
+    sk = H.lib()
+    lib = sk.load()
+    z = None
+    # decode: bad window, bad head split, unsupported head dim, B = 0 no-op
+    args = lambda B, H_q, H_kv, d, w: (z, z, z, z, z, z, 0.0, B, H_q, H_kv, d, w, 0, 0, 0, z, 0,  # noqa: E731
+                                       sk.BF16, z)
+    assert lib.speechkv_decode_attn(*args(1, 8, 4, 128, 0)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_decode_attn(*args(1, 7, 4, 128, 4)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_decode_attn(*args(1, 8, 4, 96, 4)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_decode_attn(*args(0, 8, 4, 128, 4)) == sk.OK
+    assert lib.speechkv_decode_attn(*args(1, 8, 4, 128, 4)) == sk.ERR_INVALID_ARG  # NULLs
+    # append / pool
+    assert lib.speechkv_append(z, z, z, z, z, z, 1, 8, 128, 4, -1, 0, sk.BF16, z) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_append(z, z, z, z, z, z, 0, 8, 128, 4, 0, 0, sk.BF16, z) == sk.OK
+    assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 128, 0, 0, 0, sk.BF16, z) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 80, 4, 0, 0, sk.BF16, z) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_pool(*([z] * 11), 0, 0, 8, 128, 4, 0, 0, sk.BF16, z) == sk.OK
+
+
+def test_workspace_size_explicit_grid():
+    sk = H.lib()
+    lib = sk.load()
+    B, H_q, H_kv, d, grid = 8, 16, 8, 128, 152
+    n = lib.speechkv_decode_workspace_size(B, H_q, H_kv, d, grid)
+    slot = 2 * 2 + 2 * 128
+    assert n == 256 + (grid + B * H_kv) * slot * 4
+    assert lib.speechkv_decode_workspace_size(B, 7, H_kv, d, grid) == 0
+    assert lib.speechkv_decode_workspace_size(B, H_q, H_kv, 100, grid) == 0

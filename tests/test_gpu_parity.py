@@ -1,0 +1,351 @@
+"""GPU parity: libspeechkv's kernels against the CPU oracle, element by
+element, on the same seeded inputs (paper Sec. III-B, Eq. (pool) and
+Eq. (attn); Sec. III-C for the prefill-once / append-per-step cache).
+
+Tolerances: fp32 max-abs 1e-5; bf16 max-abs 2e-2 and mean-abs 2e-3 on
+unit-variance inputs; lengths, offsets and copied rows bit-exact.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2607_06827_gb300 import inputs
+from tests import harness as H
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def sk():
+    H.require_gpu()
+    return H.lib()
+
+
+def _wl(dtype="bf16", P=(0,), T=(37,), N=(5,), G=None, w=4, l0=0, H_q=4, H_kv=2, d=64,
+        seed=7, name="case"):
+    G = G if G is not None else (0,) * len(T)
+    return inputs.Workload(name, dtype, L=1, l0=l0, w=w, H_q=H_q, H_kv=H_kv, d=d, P=list(P),
+                           T=list(T), N=list(N), G=list(G), steps=4, seed=seed)
+
+
+def _ws(sk, wl, grid=0):
+    return sk.new_workspace(wl.B, wl.H_q, wl.H_kv, wl.d, grid)
+
+
+def _decode(sk, wl, L, q, layer, grid=0, ws=None, scale=0.0):
+    out = torch.empty_like(q)
+    ws = ws if ws is not None else _ws(sk, wl, grid)
+    sk.decode_attn(q, L.k, L.v, L.cache_off, L.len, out, ws, wl.w, layer, wl.l0, wl.H_kv,
+                   scale=scale, grid_ctas=grid)
+    return out
+
+
+def _oracle_attn_on_gpu_cache(oracle, wl, L, q, scale=0.0):
+    """Oracle attention over the GPU's own cache rows (isolates the kernel)."""
+    store = oracle.STORE_F32 if wl.dtype == "f32" else oracle.STORE_BF16
+    qn = H.f64(q)
+    res = []
+    for b in range(wl.B):
+        K, V = L.request_rows(b)
+        res.append(oracle.decode_attn_request(qn[b], K, V, scale=scale, storage=store))
+    return np.stack(res)
+
+
+# --------------------------------------------------------------------------
+# pool
+# --------------------------------------------------------------------------
+POOL_CASES = [
+    # dtype, d, H_kv, P, T, N, w
+    ("f32", 64, 2, (16,), (64,), (0,), 4),            # tiny workload shapes
+    ("bf16", 128, 8, (0,), (375,), (32,), 4),         # 30 s audio, 94 entries
+    ("bf16", 128, 8, (0, 3, 0), (375, 10, 0), (32, 1, 4), 4),  # ragged, T=0
+    ("bf16", 128, 8, (2,), (13,), (3,), 3),           # T mod w != 0
+    ("bf16", 128, 8, (1,), (3,), (2,), 4),            # T < w
+    ("bf16", 64, 4, (0, 5), (40, 41), (8, 0), 8),
+    ("f32", 128, 2, (0,), (50,), (6,), 2),
+    ("bf16", 128, 8, (0,), (17,), (2,), 1),           # w = 1: bit-exact copy
+]
+
+
+@pytest.mark.parametrize("dtype,d,H_kv,P,T,N,w", POOL_CASES)
+def test_pool_matches_oracle(sk, oracle, dtype, d, H_kv, P, T, N, w):
+    wl = _wl(dtype, P, T, N, w=w, H_q=2 * H_kv, H_kv=H_kv, d=d)
+    layer = 0
+    L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=3)
+    lens = L.len.cpu().numpy()
+    for b in range(wl.B):
+        want_len = oracle.compressed_len(P[b], T[b], N[b], 0, w, layer, wl.l0)
+        assert lens[b] == want_len                          # bit-exact bookkeeping
+        Ko, Vo = oracle.pool_request(H.f64(ks[b]), H.f64(vs[b]), P[b], T[b], N[b],
+                                     H.f64(gate), w, layer, wl.l0)
+        K, V = L.request_rows(b)
+        H.assert_close(K, Ko, dtype, f"pooled K, request {b}")
+        H.assert_close(V, Vo, dtype, f"pooled V, request {b}")
+        # text rows (and every row when w = 1) are copied bit-exactly
+        n = want_len - P[b] - N[b]
+        src = H.f64(ks[b])
+        np.testing.assert_array_equal(K[:P[b]], src[:P[b]])
+        np.testing.assert_array_equal(K[P[b] + n:], src[P[b] + T[b]:])
+        if w == 1:
+            np.testing.assert_array_equal(K, src)
+            np.testing.assert_array_equal(V, H.f64(vs[b]))
+
+
+def test_pool_before_l0_is_bit_exact_copy(sk):
+    wl = _wl("bf16", (3,), (50,), (4,), w=4, l0=5, H_q=16, H_kv=8, d=128)
+    L, (ks, vs, _) = H.gpu_prefill(wl, layer=4, extra_rows=0)
+    assert int(L.len[0]) == 57
+    K, V = L.request_rows(0)
+    np.testing.assert_array_equal(K, H.f64(ks[0]))
+    np.testing.assert_array_equal(V, H.f64(vs[0]))
+
+
+def test_pool_zero_gate_is_window_mean(sk):
+    wl = _wl("f32", (0,), (30,), (0,), w=4, H_q=4, H_kv=2, d=64)
+    L, (ks, vs, _) = H.gpu_prefill(wl, 0, extra_rows=0, gate_scale=0.0)
+    K, _ = L.request_rows(0)
+    src = H.f64(ks[0])
+    for i in range(8):
+        np.testing.assert_allclose(K[i], src[4 * i:4 * i + 4].mean(axis=0), atol=1e-6)
+
+
+def test_pool_peaked_gate(sk, oracle):
+    """Large gate scale: near one-hot window weights stay finite and correct."""
+    wl = _wl("bf16", (0,), (64,), (0,), w=8, H_q=16, H_kv=8, d=128)
+    L, (ks, vs, gate) = H.gpu_prefill(wl, 0, extra_rows=0, gate_scale=1e3)
+    K, V = L.request_rows(0)
+    Ko, Vo = oracle.pool_request(H.f64(ks[0]), H.f64(vs[0]), 0, 64, 0, H.f64(gate), 8, 0, 0)
+    H.assert_close(K, Ko, "bf16", "K")
+    H.assert_close(V, Vo, "bf16", "V")
+
+
+# --------------------------------------------------------------------------
+# append
+# --------------------------------------------------------------------------
+def test_append_bit_exact_and_capacity(sk, oracle):
+    wl = _wl("bf16", (0, 2, 1), (9, 0, 4), (1, 3, 0), w=4, H_q=16, H_kv=8, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=2)
+    before_k = [L.request_rows(b, L.cap[b]) for b in range(wl.B)]
+    lens0 = L.len.cpu().numpy().copy()
+    for step in range(2):
+        _, kn, vn = inputs.step_qkv(wl, 0, step)
+        sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, 0, wl.l0)
+        assert (L.len.cpu().numpy() == lens0 + step + 1).all()
+        for b in range(wl.B):
+            K, V = L.request_rows(b)
+            np.testing.assert_array_equal(K[-1], H.f64(kn[b]))
+            np.testing.assert_array_equal(V[-1], H.f64(vn[b]))
+            np.testing.assert_array_equal(K[:-1], before_k[b][0][:K.shape[0] - 1])
+    assert sk.check_device_error() == sk.OK
+    # every cache is now full: a third append writes nothing and reports it
+    snap = (L.k.clone(), L.v.clone(), L.len.clone())
+    _, kn, vn = inputs.step_qkv(wl, 0, 9)
+    sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, 0, wl.l0)
+    assert sk.check_device_error() == sk.ERR_CAPACITY
+    assert sk.check_device_error() == sk.OK     # cleared by the read
+    assert torch.equal(L.k, snap[0]) and torch.equal(L.v, snap[1])
+    assert torch.equal(L.len, snap[2])
+
+
+# --------------------------------------------------------------------------
+# decode attention on the GPU's own cache
+# --------------------------------------------------------------------------
+ATTN_CASES = [
+    # dtype, d, H_q, H_kv, P, T, N, G, w
+    ("f32", 64, 4, 2, (16,), (64,), (0,), (8,), 4),
+    ("f32", 128, 8, 2, (0,), (300,), (7,), (0,), 4),
+    ("bf16", 128, 16, 8, (0,), (375,), (32,), (0,), 4),
+    ("bf16", 128, 16, 8, (0,), (375,), (32,), (0,), 1),
+    ("bf16", 128, 16, 16, (0, 1), (100, 7), (3, 2), (5, 0), 4),   # group 1
+    ("bf16", 128, 16, 4, (0,), (500,), (20,), (3,), 8),           # group 4
+    ("bf16", 64, 8, 4, (0, 0, 4), (63, 1500, 0), (16, 256, 9), (0, 512, 3), 4),
+    ("f32", 64, 16, 4, (2,), (33,), (1,), (0,), 2),
+]
+
+
+@pytest.mark.parametrize("dtype,d,H_q,H_kv,P,T,N,G,w", ATTN_CASES)
+def test_decode_attn_matches_oracle(sk, oracle, dtype, d, H_q, H_kv, P, T, N, G, w):
+    wl = _wl(dtype, P, T, N, G, w=w, H_q=H_q, H_kv=H_kv, d=d)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=0)
+    q, _, _ = inputs.step_qkv(wl, 0, 0)
+    q = q.cuda()
+    ref = _oracle_attn_on_gpu_cache(oracle, wl, L, q)
+    for grid in (0, 1, 2, 7, 300):
+        out = _decode(sk, wl, L, q, 0, grid=grid)
+        H.assert_close(H.f64(out), ref, dtype, f"decode attn, grid {grid}")
+    assert sk.check_device_error() == sk.OK
+
+
+def test_decode_attn_ragged_batch_invariance(sk, oracle):
+    """A request's output in a ragged batch matches the same request alone."""
+    wl = _wl("bf16", (0,) * 5, (63, 900, 1, 250, 1500), (16, 100, 200, 3, 30),
+             (0, 7, 512, 0, 100), w=4, H_q=16, H_kv=8, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=0)
+    q = inputs.step_qkv(wl, 0, 0)[0].cuda()
+    full = _decode(sk, wl, L, q, 0)
+    for b in (1, 4):
+        one = _wl("bf16", (0,), (wl.T[b],), (wl.N[b],), (wl.G[b],), w=4, H_q=16, H_kv=8, d=128)
+        L1 = H.GpuLayer(one, 0, 0)
+        K, V = L.block(L.k, b), L.block(L.v, b)
+        L1.block(L1.k, 0).copy_(K)
+        L1.block(L1.v, 0).copy_(V)
+        L1.len.copy_(L.len[b:b + 1])
+        out1 = _decode(sk, one, L1, q[b:b + 1].contiguous(), 0)
+        H.assert_close(H.f64(out1[0]), H.f64(full[b]), "bf16", f"request {b} alone")
+
+
+def test_decode_attn_edge_cases(sk, oracle):
+    wl = _wl("bf16", (0, 0, 0), (8, 16, 4), (0, 2, 0), w=4, H_q=8, H_kv=4, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=4)
+    q = inputs.step_qkv(wl, 0, 0)[0].cuda()
+    # an empty request gets zeros; the others are unaffected
+    L.len[1] = 0
+    out = _decode(sk, wl, L, q, 0)
+    assert not out[1].any()
+    ref = _oracle_attn_on_gpu_cache(oracle, wl, L, q)
+    H.assert_close(H.f64(out), ref, "bf16", "with an empty request")
+    # all empty
+    L.len.zero_()
+    assert not _decode(sk, wl, L, q, 0).any()
+    # a length beyond capacity is reported and clamped
+    L.len.copy_(torch.tensor([1, 2, 100], dtype=torch.int32))
+    out = _decode(sk, wl, L, q, 0)
+    assert sk.check_device_error() == sk.ERR_CAPACITY
+    L.len[2] = L.cap[2]
+    ref = _oracle_attn_on_gpu_cache(oracle, wl, L, q)
+    H.assert_close(H.f64(out), ref, "bf16", "clamped length")
+    # a single cached row returns its value exactly (up to the output rounding)
+    L.len.fill_(1)
+    out = _decode(sk, wl, L, q, 0)
+    for b in range(wl.B):
+        _, V = L.request_rows(b)
+        for hq in range(wl.H_q):
+            np.testing.assert_array_equal(H.f64(out[b, hq]), V[0, hq // 2])
+    # B = 0 is a no-op
+    empty = torch.empty((0, 8, 128), dtype=torch.bfloat16, device="cuda")
+    sk.decode_attn(empty, L.k, L.v, L.cache_off, L.len[:0], empty, _ws(sk, wl), 4, 0, 0, 4)
+    assert sk.check_device_error() == sk.OK
+
+
+def test_decode_attn_extreme_logits(sk, oracle):
+    wl = _wl("bf16", (0,), (600,), (10,), w=4, H_q=16, H_kv=8, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=0)
+    q = (inputs.step_qkv(wl, 0, 0)[0].float() * 100).to(torch.bfloat16).cuda()
+    out = _decode(sk, wl, L, q, 0)
+    assert torch.isfinite(out.float()).all()
+    H.assert_close(H.f64(out), _oracle_attn_on_gpu_cache(oracle, wl, L, q), "bf16", "q x 100")
+
+
+def test_decode_attn_explicit_scale(sk, oracle):
+    wl = _wl("f32", (0,), (100,), (4,), w=4, H_q=4, H_kv=2, d=64)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=0)
+    q = inputs.step_qkv(wl, 0, 0)[0].cuda()
+    out = _decode(sk, wl, L, q, 0, scale=0.05)
+    H.assert_close(H.f64(out), _oracle_attn_on_gpu_cache(oracle, wl, L, q, scale=0.05), "f32",
+                   "scale 0.05")
+
+
+def test_invalid_arguments_return_status(sk):
+    wl = _wl("bf16", (0,), (8,), (0,), w=4, H_q=8, H_kv=4, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=1)
+    q = inputs.step_qkv(wl, 0, 0)[0].cuda()
+    out = torch.empty_like(q)
+    ws = _ws(sk, wl)
+    lib = sk.load()
+    common = (q.data_ptr(), L.k.data_ptr(), L.v.data_ptr(), L.cache_off.data_ptr(),
+              L.len.data_ptr(), out.data_ptr(), 0.0)
+    s = torch.cuda.current_stream().cuda_stream
+    nbytes = ws.numel()
+
+    def call(B=1, H_q=8, H_kv=4, d=128, w=4, grid=0, wsb=nbytes, dt=sk.BF16, p=common):
+        return lib.speechkv_decode_attn(*p, B, H_q, H_kv, d, w, 0, 0, grid, ws.data_ptr(), wsb,
+                                        dt, s)
+    assert call() == sk.OK
+    assert call(w=0) == sk.ERR_INVALID_ARG
+    assert call(H_q=7) == sk.ERR_INVALID_ARG
+    assert call(d=96) == sk.ERR_UNSUPPORTED
+    assert call(H_q=32, H_kv=4) == sk.ERR_UNSUPPORTED       # group 8 not built
+    assert call(B=sk.MAX_BATCH + 1) == sk.ERR_UNSUPPORTED
+    assert call(wsb=16) == sk.ERR_WORKSPACE
+    assert call(grid=-1) == sk.ERR_INVALID_ARG
+    misaligned = (q.data_ptr() + 2,) + common[1:]
+    assert call(p=misaligned) == sk.ERR_INVALID_ARG
+    nullq = (None,) + common[1:]
+    assert call(p=nullq) == sk.ERR_INVALID_ARG
+    assert sk.check_device_error() == sk.OK
+
+
+# --------------------------------------------------------------------------
+# whole path: prefill pooling, then append + attend for several steps
+# --------------------------------------------------------------------------
+def _run_steps(sk, oracle, wl, layers, steps):
+    for layer in layers:
+        L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=steps)
+        oc = H.oracle_prefill(oracle, wl, layer, steps, ks, vs, gate)
+        ws = _ws(sk, wl)
+        store = oracle.STORE_F32 if wl.dtype == "f32" else oracle.STORE_BF16
+        for b in range(wl.B):
+            assert int(L.len[b]) == oc[b][2]
+        for step in range(steps):
+            q, kn, vn = inputs.step_qkv(wl, layer, step)
+            sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
+            out = _decode(sk, wl, L, q.cuda(), layer, ws=ws)
+            ref = []
+            for b in range(wl.B):
+                Kc, Vc, n = oc[b]
+                n = oracle.append_request(Kc, Vc, n, H.f64(kn[b]), H.f64(vn[b]))
+                oc[b][2] = n
+                assert int(L.len[b]) == n
+                ref.append(oracle.decode_attn_request(H.f64(q[b]), Kc[:n], Vc[:n],
+                                                      storage=store))
+            H.assert_close(H.f64(out), np.stack(ref), wl.dtype, f"layer {layer} step {step}")
+    assert sk.check_device_error() == sk.OK
+
+
+def test_end_to_end_tiny_fp32(sk, oracle):
+    """Tiny fp32 workload: 16 text + 64 frames (w=4 -> 16 entries), 8 steps;
+    cached rows go 33 -> 40."""
+    _run_steps(sk, oracle, inputs.tiny_fp32(), layers=[0], steps=8)
+
+
+def test_end_to_end_qwen_single(sk, oracle):
+    """Qwen3-1.7B shapes, 30 s audio: one layer before l0 (full resolution)
+    and one pooled layer, first 6 of the 128 steps."""
+    wl = inputs.qwen_single()
+    _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=6)
+
+
+def test_end_to_end_ragged_small(sk, oracle):
+    wl = inputs.qwen_ragged(B=6)
+    _run_steps(sk, oracle, wl, layers=[wl.l0], steps=3)
+
+
+# --------------------------------------------------------------------------
+# full benchmark sizes, sampled against the oracle
+# --------------------------------------------------------------------------
+def _sampled_full_size(sk, oracle, wl, layer, samples):
+    L, _ = H.gpu_prefill(wl, layer, extra_rows=1)
+    q, kn, vn = inputs.step_qkv(wl, layer, 0)
+    sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
+    out = _decode(sk, wl, L, q.cuda(), layer)
+    assert sk.check_device_error() == sk.OK
+    lens = L.len.cpu().numpy()
+    for b in samples:
+        assert lens[b] == oracle.compressed_len(wl.P[b], wl.T[b], wl.N[b], wl.G[b] + 1, wl.w,
+                                                layer, wl.l0)
+        K, V = L.request_rows(b)
+        ref = oracle.decode_attn_request(H.f64(q[b]), K, V, storage=oracle.STORE_BF16)
+        H.assert_close(H.f64(out[b]), ref, "bf16", f"request {b}")
+
+
+@pytest.mark.parametrize("minutes,w", [(20, 4), (10, 8)])
+def test_full_size_long_audio_sampled(sk, oracle, minutes, w):
+    wl = inputs.qwen_long_audio(minutes, w, generated=64)
+    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 5])
+
+
+def test_full_size_ragged_sampled(sk, oracle):
+    wl = inputs.qwen_ragged()
+    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 17, 64, 127])
