@@ -127,17 +127,22 @@ def test_pool_peaked_gate(sk, oracle):
 def test_append_bit_exact_and_capacity(sk, oracle):
     wl = _wl("bf16", (0, 2, 1), (9, 0, 4), (1, 3, 0), w=4, H_q=16, H_kv=8, d=128)
     L, _ = H.gpu_prefill(wl, 0, extra_rows=2)
-    before_k = [L.request_rows(b, L.cap[b]) for b in range(wl.B)]
     lens0 = L.len.cpu().numpy().copy()
+    before = [L.request_rows(b) for b in range(wl.B)]
+    added_k, added_v = [], []
     for step in range(2):
         _, kn, vn = inputs.step_qkv(wl, 0, step)
         sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, 0, wl.l0)
+        added_k.append(H.f64(kn)); added_v.append(H.f64(vn))
         assert (L.len.cpu().numpy() == lens0 + step + 1).all()
         for b in range(wl.B):
             K, V = L.request_rows(b)
-            np.testing.assert_array_equal(K[-1], H.f64(kn[b]))
-            np.testing.assert_array_equal(V[-1], H.f64(vn[b]))
-            np.testing.assert_array_equal(K[:-1], before_k[b][0][:K.shape[0] - 1])
+            n0 = lens0[b]
+            np.testing.assert_array_equal(K[:n0], before[b][0])
+            np.testing.assert_array_equal(V[:n0], before[b][1])
+            for j in range(step + 1):
+                np.testing.assert_array_equal(K[n0 + j], added_k[j][b])
+                np.testing.assert_array_equal(V[n0 + j], added_v[j][b])
     assert sk.check_device_error() == sk.OK
     # every cache is now full: a third append writes nothing and reports it
     snap = (L.k.clone(), L.v.clone(), L.len.clone())
