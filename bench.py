@@ -69,6 +69,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="budget of the oracle CPU baseline sample")
     ap.add_argument("--graph-chunk", type=int, default=32)
+    ap.add_argument("--layers", type=str, default=None,
+                    help="comma-separated layer indices to build (default: all 28); "
+                         "for small profiling cases only")
     return ap.parse_args()
 
 
@@ -169,12 +172,14 @@ class ClockSampler:
 class DecodeModel:
     """Per-layer caches built by speechkv_pool, per-step inputs resident in HBM."""
 
-    def __init__(self, wl, steps_total: int, seed_key: int, device="cuda"):
+    def __init__(self, wl, steps_total: int, seed_key: int, device="cuda", layers=None):
         import torch
         from paper_2607_06827_gb300 import inputs, speechkv as sk
         self.wl, self.sk, self.device = wl, sk, device
+        self.layers = list(layers) if layers is not None else list(range(wl.L))
         self.dtype = torch.bfloat16
-        B, Hq, Hk, d, L = wl.B, wl.H_q, wl.H_kv, wl.d, wl.L
+        B, Hq, Hk, d = wl.B, wl.H_q, wl.H_kv, wl.d
+        L = len(self.layers)
         full_rows = sum(wl.full_rows())
         full_off = [0]
         for s in wl.full_rows():
@@ -184,7 +189,7 @@ class DecodeModel:
         full_off_t = torch.tensor(full_off, dtype=torch.int64, device=device)
         self.k, self.v, self.len, self.off, self.rows0 = [], [], [], [], []
         self.pool_ms = {}
-        for layer in range(L):
+        for layer in self.layers:
             cap = [sk.compressed_len(wl.P[b], wl.T[b], wl.N[b], wl.G[b], wl.w, layer, wl.l0)
                    + steps_total for b in range(B)]
             off = [0]
@@ -213,10 +218,10 @@ class DecodeModel:
             for g in range(wl.G[0]):
                 kn = inputs.device_normal((L, B, Hk, d), self.dtype, device, wl.seed, seed_key, 4, g)
                 vn = inputs.device_normal((L, B, Hk, d), self.dtype, device, wl.seed, seed_key, 5, g)
-                for layer in range(L):
-                    sk.append(kn[layer], vn[layer], self.k[layer], self.v[layer], self.off[layer],
-                              self.len[layer], wl.w, layer, wl.l0)
-        self.rows0 = [self.len[layer].cpu().tolist() for layer in range(L)]
+                for i, layer in enumerate(self.layers):
+                    sk.append(kn[i], vn[i], self.k[i], self.v[i], self.off[i], self.len[i],
+                              wl.w, layer, wl.l0)
+        self.rows0 = [self.len[i].cpu().tolist() for i in range(L)]
         # per-step inputs, resident before the timed region
         self.q = inputs.device_normal((steps_total, L, B, Hq, d), self.dtype, device, wl.seed, seed_key, 6)
         self.kn = inputs.device_normal((steps_total, L, B, Hk, d), self.dtype, device, wl.seed, seed_key, 7)
@@ -228,18 +233,17 @@ class DecodeModel:
 
     def launch_step(self, s: int, events=None):
         wl, sk = self.wl, self.sk
-        for layer in range(wl.L):
-            sk.append(self.kn[s, layer], self.vn[s, layer], self.k[layer], self.v[layer],
-                      self.off[layer], self.len[layer], wl.w, layer, wl.l0)
+        for i, layer in enumerate(self.layers):
+            sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
+                      self.len[i], wl.w, layer, wl.l0)
             if events is not None:
-                events[layer][0].record()
-            sk.decode_attn(self.q[s, layer], self.k[layer], self.v[layer], self.off[layer],
-                           self.len[layer], self.out[layer], self.ws, wl.w, layer, wl.l0,
-                           wl.H_kv)
+                events[i][0].record()
+            sk.decode_attn(self.q[s, i], self.k[i], self.v[i], self.off[i], self.len[i],
+                           self.out[i], self.ws, wl.w, layer, wl.l0, wl.H_kv)
             if events is not None:
-                events[layer][1].record()
+                events[i][1].record()
 
-    def attn_bytes(self, layer: int, rows_per_req) -> int:
+    def attn_bytes(self, rows_per_req) -> int:
         """Algorithmic bytes of one decode_attn launch: every cached K and V
         row once, the queries and the outputs (bf16)."""
         wl = self.wl
@@ -256,7 +260,7 @@ def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist:
     """Capture `steps` decode steps in CUDA graphs of `chunk` steps, then replay
     them as the timed region.  Returns (region_ms, per-layer attn ms lists)."""
     import torch
-    L = model.wl.L
+    L = len(model.layers)
     graphs, evs = [], []
     s = first_step
     while s < first_step + steps:
@@ -294,29 +298,30 @@ def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist:
 
 
 def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int,
-            keep_model=False):
+            layers=None):
     """Build the model for `wl`, run warm-up steps eagerly, time `steps`
-    graph-replayed steps.  Returns a result dict (and the model if asked)."""
+    graph-replayed steps.  Returns a result dict."""
     import torch
-    model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key)
+    model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key, layers=layers)
     for s in range(warmup):
         model.launch_step(s)
     torch.cuda.synchronize()
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
-    base_rows = [[model.rows0[layer][b] + warmup for b in range(wl.B)] for layer in range(wl.L)]
+    L = len(model.layers)
+    base_rows = [[model.rows0[i][b] + warmup for b in range(wl.B)] for i in range(L)]
     region_ms, per_layer = run_timed(model, warmup, steps, chunk, dist, clocks)
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
-    L = wl.L
-    comp = [l for l in range(L) if l >= wl.l0]
-    full = [l for l in range(L) if l < wl.l0]
+    comp = [i for i, layer in enumerate(model.layers) if layer >= wl.l0]
+    full = [i for i, layer in enumerate(model.layers) if layer < wl.l0]
     mean = lambda xs: sum(xs) / len(xs) if xs else float("nan")  # noqa: E731
-    attn_ms = {l: mean(per_layer[l]) for l in range(L)}
+    ratio = lambda a, b: a / b if b else float("nan")  # noqa: E731
+    attn_ms = {i: mean(per_layer[i]) for i in range(L)}
     # algorithmic bytes: rows after step t's append are base + t + 1
-    bytes_total = {l: sum(model.attn_bytes(l, [r + t + 1 for r in base_rows[l]])
-                          for t in range(steps)) for l in range(L)}
-    time_total = {l: sum(per_layer[l]) for l in range(L)}
+    bytes_total = {i: sum(model.attn_bytes([r + t + 1 for r in base_rows[i]])
+                          for t in range(steps)) for i in range(L)}
+    time_total = {i: sum(per_layer[i]) for i in range(L)}
     res = {
         "minutes": wl.T[0] * 80 / 60000.0, "w": wl.w, "B": wl.B,
         "step_us": region_ms * 1e3 / steps,
@@ -324,30 +329,31 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
         "attn_us_per_layer": mean([attn_ms[l] for l in range(L)]) * 1e3,
         "attn_us_compressed_layer": mean([attn_ms[l] for l in comp]) * 1e3,
         "attn_us_full_layer": mean([attn_ms[l] for l in full]) * 1e3,
-        "attn_gbs_compressed_layer": (sum(bytes_total[l] for l in comp) /
-                                      (sum(time_total[l] for l in comp) * 1e-3) / 1e9),
-        "attn_gbs_all_layers": (sum(bytes_total.values()) / (sum(time_total.values()) * 1e-3) / 1e9),
-        "attn_bytes_per_launch_compressed": sum(bytes_total[l] for l in comp) / (len(comp) * steps),
+        "attn_gbs_compressed_layer": ratio(sum(bytes_total[i] for i in comp),
+                                           sum(time_total[i] for i in comp) * 1e-3) / 1e9,
+        "attn_gbs_all_layers": ratio(sum(bytes_total.values()),
+                                     sum(time_total.values()) * 1e-3) / 1e9,
+        "attn_bytes_per_launch_compressed": ratio(sum(bytes_total[i] for i in comp),
+                                                  len(comp) * steps),
         "attn_bytes_per_launch_all": sum(bytes_total.values()) / (L * steps),
-        "pool_us_compressed_layer": mean([model.pool_ms[l] for l in comp]) * 1e3,
-        "pool_us_full_layer": mean([model.pool_ms[l] for l in full]) * 1e3,
+        "pool_us_compressed_layer": mean([model.pool_ms[model.layers[i]] for i in comp]) * 1e3,
+        "pool_us_full_layer": mean([model.pool_ms[model.layers[i]] for i in full]) * 1e3,
         "gpu_launches": steps * L * 2,
         "region_ms": region_ms,
     }
-    if keep_model:
-        return res, model
     model.free()
     del model
     torch.cuda.empty_cache()
     return res
 
 
-def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int):
+def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int,
+                layers=None):
     """Same decode steps through the C ABI with HOST buffers: every step copies
     its q/k/v from pinned host memory and reads the outputs back."""
     import torch
-    model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key)
-    L, B, Hq, Hk, d = wl.L, wl.B, wl.H_q, wl.H_kv, wl.d
+    model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key, layers=layers)
+    L, B, Hq, Hk, d = len(model.layers), wl.B, wl.H_q, wl.H_kv, wl.d
     total = warmup + steps
     h_q = model.q.cpu().pin_memory()
     h_kn = model.kn.cpu().pin_memory()
@@ -359,15 +365,15 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
     sk = model.sk
 
     def step(s):
-        for layer in range(L):
-            d_q[layer].copy_(h_q[s, layer], non_blocking=True)
-            d_kn[layer].copy_(h_kn[s, layer], non_blocking=True)
-            d_vn[layer].copy_(h_vn[s, layer], non_blocking=True)
-            sk.append(d_kn[layer], d_vn[layer], model.k[layer], model.v[layer], model.off[layer],
-                      model.len[layer], wl.w, layer, wl.l0)
-            sk.decode_attn(d_q[layer], model.k[layer], model.v[layer], model.off[layer],
-                           model.len[layer], model.out[layer], model.ws, wl.w, layer, wl.l0, Hk)
-            h_out[s, layer].copy_(model.out[layer], non_blocking=True)
+        for i, layer in enumerate(model.layers):
+            d_q[i].copy_(h_q[s, i], non_blocking=True)
+            d_kn[i].copy_(h_kn[s, i], non_blocking=True)
+            d_vn[i].copy_(h_vn[s, i], non_blocking=True)
+            sk.append(d_kn[i], d_vn[i], model.k[i], model.v[i], model.off[i], model.len[i],
+                      wl.w, layer, wl.l0)
+            sk.decode_attn(d_q[i], model.k[i], model.v[i], model.off[i], model.len[i],
+                           model.out[i], model.ws, wl.w, layer, wl.l0, Hk)
+            h_out[s, i].copy_(model.out[i], non_blocking=True)
 
     for s in range(warmup):
         step(s)
@@ -496,7 +502,7 @@ def run_reference(args):
                                     "layer, scaled to the batch and the 28-layer mix")},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
-    print(json.dumps(line), flush=True)
+    print(json.dumps(finite_json(line)), flush=True)
 
 
 # ---------------------------------------------------------------------------
@@ -513,6 +519,17 @@ def workload_config(minutes: int, w: int, n_gpus: int) -> dict:
         "l2": "no flush: per-step working set of several GB exceeds the 129 MB L2; "
               "consecutive layers read disjoint caches",
     }
+
+
+def finite_json(x):
+    """Replace NaN/inf (not valid JSON) by None, recursively."""
+    if isinstance(x, float):
+        return x if math.isfinite(x) else None
+    if isinstance(x, dict):
+        return {k: finite_json(v) for k, v in x.items()}
+    if isinstance(x, (list, tuple)):
+        return [finite_json(v) for v in x]
+    return x
 
 
 def measured_peak():
@@ -565,16 +582,19 @@ def main():
     dist = Dist(args.gpus)
     clocks = ClockSampler(dist.local) if dist.rank == 0 else None
 
+    layers = [int(x) for x in args.layers.split(",")] if args.layers else None
     wl = inputs.qwen_long_audio(args.minutes, args.w, generated=GENERATED)
-    main_res = measure(wl, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0)
+    main_res = measure(wl, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0,
+                       layers=layers)
     w1_res = None
     if not args.no_w1:
         wl1 = inputs.qwen_long_audio(args.minutes, 1, generated=GENERATED)
-        w1_res = measure(wl1, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0)
+        w1_res = measure(wl1, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0,
+                         layers=layers)
     e2e = None
     if not args.no_e2e:
         e2e = measure_e2e(wl, min(args.e2e_steps, args.steps), args.warmup, args.graph_chunk,
-                          dist, clocks, seed_key=0)
+                          dist, clocks, seed_key=0, layers=layers)
     sweep = []
     if not args.no_sweep:
         done = {(args.minutes, args.w): main_res}
@@ -583,12 +603,13 @@ def main():
             if (minutes, w) in done:
                 continue
             r = measure(inputs.qwen_long_audio(minutes, w, generated=GENERATED),
-                        args.sweep_steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0)
+                        args.sweep_steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0,
+                        layers=layers)
             done[(minutes, w)] = r
             if minutes not in w1_by_min:
                 w1_by_min[minutes] = measure(
                     inputs.qwen_long_audio(minutes, 1, generated=GENERATED), args.sweep_steps,
-                    args.warmup, args.graph_chunk, dist, clocks, seed_key=0)
+                    args.warmup, args.graph_chunk, dist, clocks, seed_key=0, layers=layers)
         for (minutes, w), r in sorted(done.items()):
             w1 = w1_by_min.get(minutes)
             sweep.append({
@@ -657,7 +678,7 @@ def main():
             } if w1_res else None),
             "by_audio_len": sweep or None,
         }
-        print(json.dumps(line), flush=True)
+        print(json.dumps(finite_json(line)), flush=True)
     dist.close()
 
 

@@ -66,7 +66,7 @@ typedef enum {
 typedef enum { SPEECHKV_F32 = 0, SPEECHKV_BF16 = 1 } speechkv_dtype;
 
 /* Largest batch speechkv_decode_attn accepts (its per-CTA length table). */
-#define SPEECHKV_MAX_BATCH 2048
+#define SPEECHKV_MAX_BATCH 1024
 
 /* Human-readable name of a status (static string, never NULL). */
 const char *speechkv_status_string(speechkv_status status);

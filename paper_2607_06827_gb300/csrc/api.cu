@@ -18,11 +18,13 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 constexpr int kDecodeKinds = 12;  // dtype x d x group
+constexpr int kBatchBuckets = 3;  // occupancy is cached per batch-size bucket
+constexpr int kBatchBucketMax[kBatchBuckets] = {128, 512, SPEECHKV_MAX_BATCH};
 
 struct DeviceState {
     int *err = nullptr;  // device address of speechkv_error_word
     int num_sms = 0;
-    int decode_ctas_per_sm[kDecodeKinds] = {};
+    int decode_ctas_per_sm[kDecodeKinds][kBatchBuckets] = {};
 };
 
 std::mutex g_mu;
@@ -68,24 +70,27 @@ int decode_kind(speechkv_dtype dt, int d, int group) {
     return (dt == SPEECHKV_BF16 ? 6 : 0) + (d == 128 ? 3 : 0) + g;
 }
 
-// Automatic decode grid: one CTA per SM times the kernel's residency (at most
-// two).  Workspace sizing uses the upper bound kAutoCtasPerSmMax.
-constexpr int kAutoCtasPerSmMax = 2;
+// Automatic decode grid: the SM count times the kernel's residency (which
+// depends on the batch size through the per-CTA length table), at most
+// kAutoCtasPerSmMax.  Workspace sizing uses that upper bound.
+constexpr int kAutoCtasPerSmMax = 4;
 
-speechkv_status decode_auto_grid(DeviceState *s, speechkv_dtype dt, int d, int group,
+speechkv_status decode_auto_grid(DeviceState *s, speechkv_dtype dt, int d, int group, int B,
                                  int *grid) {
     const int kind = decode_kind(dt, d, group);
+    int bucket = 0;
+    while (bucket < kBatchBuckets - 1 && B > kBatchBucketMax[bucket]) bucket++;
     int per_sm;
     {
         std::lock_guard<std::mutex> lock(g_mu);
-        per_sm = s->decode_ctas_per_sm[kind];
+        per_sm = s->decode_ctas_per_sm[kind][bucket];
     }
     if (per_sm == 0) {
-        per_sm = speechkv::decode_ctas_per_sm(dt, d, group);
+        per_sm = speechkv::decode_ctas_per_sm(dt, d, group, kBatchBucketMax[bucket]);
         if (per_sm <= 0) return SPEECHKV_ERR_CUDA;
         if (per_sm > kAutoCtasPerSmMax) per_sm = kAutoCtasPerSmMax;
         std::lock_guard<std::mutex> lock(g_mu);
-        s->decode_ctas_per_sm[kind] = per_sm;
+        s->decode_ctas_per_sm[kind][bucket] = per_sm;
     }
     *grid = s->num_sms * per_sm;
     return SPEECHKV_OK;
@@ -236,7 +241,7 @@ speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const v
     if (st != SPEECHKV_OK) return st;
     int grid = grid_ctas;
     if (grid == 0) {
-        st = decode_auto_grid(s, dtype, d, H_q / H_kv, &grid);
+        st = decode_auto_grid(s, dtype, d, H_q / H_kv, B, &grid);
         if (st != SPEECHKV_OK) return st;
     }
     const size_t need = workspace_bytes(B, H_q, H_kv, d, grid);

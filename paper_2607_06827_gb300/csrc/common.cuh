@@ -138,6 +138,65 @@ __device__ __forceinline__ float fast_exp2(float x) {
 }
 
 // ---------------------------------------------------------------------------
+// packed fp32 pairs (sm_100+ f32x2 arithmetic: two lanes of math per issue)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+// The two bf16 of a packed 32-bit word as an fp32 pair (exact).
+__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t x) {
+    return make_float2(bf16_lo(x), bf16_hi(x));
+}
+
+// 16 bytes of T as fp32 pairs: 4 pairs for bf16, 2 for fp32.
+template <typename T>
+__device__ __forceinline__ void load16_pairs(const void *p, float2 (&f)[16 / sizeof(T) / 2]) {
+    if constexpr (sizeof(T) == 2) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(p);
+        f[0] = bf16x2_to_float2(v.x);
+        f[1] = bf16x2_to_float2(v.y);
+        f[2] = bf16x2_to_float2(v.z);
+        f[3] = bf16x2_to_float2(v.w);
+    } else {
+        const float4 v = *reinterpret_cast<const float4 *>(p);
+        f[0] = make_float2(v.x, v.y);
+        f[1] = make_float2(v.z, v.w);
+    }
+}
+
+// Atomic add with acquire-release semantics at GPU scope (publishes the
+// CTA's earlier writes, ordered before it by a barrier, to the acquirer).
+__device__ __forceinline__ int atomic_add_acq_rel_gpu(int *p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v)
+                 : "memory");
+    return old;
+}
+
+// Orders this thread's earlier generic-proxy shared-memory accesses before
+// later async-proxy (TMA) accesses of the same shared memory.
+__device__ __forceinline__ void fence_proxy_async_shared() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
 // mbarrier + bulk asynchronous copy (TMA, non-tensor form)
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {

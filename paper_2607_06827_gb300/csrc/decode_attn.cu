@@ -2,26 +2,32 @@
 // step -- every query head attends over its request's cached (pooled speech
 // + text) keys and values, grouped-query style.
 //
-// Design (GB300, HBM-bound):
+// Design (GB300, HBM-bound, about 2 flop per byte):
 //   * Work = sum over requests of len[b] rows times H_kv heads.  A persistent
-//     grid cuts this flat range evenly (stream-K): CTA c owns units
-//     [U*c/C, U*(c+1)/C).  Its range splits into "pieces", each a run of rows
-//     of one (request, KV head).  Every CTA therefore reads the same number of
-//     bytes whatever the length mix of the batch.
+//     grid (three small CTAs per SM) cuts this flat range evenly (stream-K):
+//     CTA c owns units [U*c/C, U*(c+1)/C), whatever the length mix of the
+//     batch.  Its range splits into "pieces", each a run of rows of one
+//     (request, KV head).
 //   * The cache is head-major per request, so a piece is one contiguous run
-//     of rows.  One producer lane streams it HBM -> shared memory with bulk
-//     asynchronous copies (TMA, cp.async.bulk) into a ring of stages guarded
-//     by mbarriers; eight consumer warps compute on the staged tiles.
+//     of rows.  One producer lane streams it HBM -> shared memory in 64-row
+//     tiles with bulk asynchronous copies (TMA, cp.async.bulk: one copy for
+//     the keys, one for the values, plus the piece's queries with its first
+//     tile) into a two-stage ring guarded by mbarriers.  Four consumer warps
+//     take 16 rows each of every tile.  Several CTAs per SM keep the memory
+//     pipe busy while one of them merges a piece.
 //   * All G = H_q/H_kv query heads of the KV head are served from one read of
 //     each key/value row.  QK: four lanes per row, each reading a quarter of
 //     the row from shared memory in an order that keeps every 8-lane phase on
-//     distinct banks, two-step shuffle reduction.  Softmax: online (running
-//     max and sum per warp) in base 2, the log2(e)/sqrt(d) factor folded into
-//     the query.  PV: each lane owns d/32 output columns of every head.
-//   * A piece that covers a whole (request, head) writes the output.  Pieces
-//     of a (request, head) split across CTAs write (max, sum, unnormalised o)
-//     partials; the CTA that arrives last (atomic ticket, no waiting) merges
-//     them with log-sum-exp weights and resets the counter for the next call.
+//     distinct banks, packed f32x2 FMAs, two-step shuffle reduction.  Softmax:
+//     online (running max and sum per warp) in base 2, with log2(e)/sqrt(d)
+//     folded into the query.  PV: each lane owns one 16-byte column chunk of
+//     a row (two rows per warp instruction for bf16, d = 128), f32x2 FMAs.
+//   * At the end of a piece the consumer warps' (max, sum, o) states are
+//     merged in shared memory.  A piece covering a whole (request, head)
+//     writes the output; otherwise it writes an unnormalised partial, and the
+//     CTA that arrives last at that (request, head) (atomic ticket with
+//     acquire-release ordering, no waiting) merges the partials with
+//     log-sum-exp weights and resets the ticket for the next call.
 //   * Every mbarrier wait is bounded; on timeout the kernel reports
 //     SPEECHKV_ERR_TIMEOUT, stops issuing and computing, lets its copies in
 //     flight land and returns.
@@ -35,37 +41,45 @@ namespace {
 
 template <typename T, int D, int G>
 struct DecodeCfg {
-    static constexpr int kWarps = 8;                    // consumer warps
-    static constexpr int kThreads = (kWarps + 1) * 32;  // + one producer warp
+    static constexpr int kWarps = 8;  // consumer warps
+    // + one producer warp (lane 0 issues the bulk copies) + one merge warp
+    static constexpr int kThreads = (kWarps + 2) * 32;
+    static constexpr int kCtasPerSm = 1;
     static constexpr int kRowBytes = D * (int)sizeof(T);
-    static constexpr int kChunks = kRowBytes / 16;      // 16-byte chunks per row
-    static constexpr int kChunksPerLane = kChunks / 4;  // QK: 4 lanes per row
-    static constexpr int kElemsPerChunk = 16 / (int)sizeof(T);
-    static constexpr int kRowsPerGroup = kRowBytes >= 512 ? 1 : 2;
-    static constexpr int kRowsPerWarp = 8 * kRowsPerGroup;
+    static constexpr int kRowsPerWarp = kRowBytes >= 512 ? 8 : 16;
     static constexpr int kTileRows = kWarps * kRowsPerWarp;
-    static constexpr int kTileBytes = kTileRows * kRowBytes;  // K (or V) of a tile
-    static constexpr int kStageBytes = 2 * kTileBytes;
-    static constexpr int kColsPerLane = D / 32;               // PV columns per lane
-    static constexpr int kMergeBytes = kWarps * G * D * 4 + 2 * kWarps * G * 4;
-    static constexpr int kPBytes = kWarps * kRowsPerWarp * G * 4;
+    static constexpr int kTileBytes = kTileRows * kRowBytes;  // keys (or values) of a tile
+    static constexpr int kQBytes = G * kRowBytes;             // the piece's G query rows
+    static constexpr int kStageBytes = 2 * kTileBytes + kQBytes;
+    // QK layout: 4 lanes per row, 8 rows per pass
+    static constexpr int kChunks = kRowBytes / 16;  // 16-byte chunks per row
+    static constexpr int kChunksPerLane = kChunks / 4;
+    static constexpr int kPairsPerChunk = 16 / (int)sizeof(T) / 2;
+    static constexpr int kQkPasses = kRowsPerWarp / 8;
+    // PV layout: one 16-byte chunk per lane, kPvRowsPerPass rows per pass
+    static constexpr int kPvLanesPerRow = kChunks;
+    static constexpr int kPvRowsPerPass = 32 / kPvLanesPerRow;
+    // shared memory: stages | barriers | p | 2 merge buffers | flags | cum
+    static constexpr int kPBytes = kWarps * kRowsPerWarp * G * 8;  // (p, p) pairs
+    static constexpr int kMergeFloats = kWarps * G * D + 2 * kWarps * G;
+    static constexpr int kMergeBytes = 2 * kMergeFloats * 4;
+    static constexpr int kBarBytes = (2 * 3 + 4) * 8;  // full/empty per stage (<= 3), piece/free x2
     static constexpr int kSmemLimit = 227 * 1024;
-    static constexpr int kCumMaxBytes = (SPEECHKV_MAX_BATCH + 1) * 8;
-    static constexpr int kFixedMax = kMergeBytes + kPBytes + 2 * 4 * 8 + 16 + kCumMaxBytes;
+    static constexpr int kFixedMax =
+        kBarBytes + kPBytes + kMergeBytes + 16 + (SPEECHKV_MAX_BATCH + 1) * 8;
     static constexpr int kStagesFit = (kSmemLimit - kFixedMax) / kStageBytes;
-    static constexpr int kStages = kStagesFit < 4 ? kStagesFit : 4;
+    static constexpr int kStages = kStagesFit < 3 ? kStagesFit : 3;
+    static constexpr int kStagesBytes = kStages * kStageBytes;
     static_assert(kStages >= 2, "shared memory too small for two stages");
+    static_assert(kStageBytes % 16 == 0 && kTileBytes % 16 == 0, "bulk copy alignment");
     static_assert(kChunksPerLane >= 2, "row too short for the QK lane layout");
+    static_assert(kPvLanesPerRow <= 32, "row too long for the PV lane layout");
 
     static size_t smem_bytes(int B) {
-        return (size_t)kStages * kStageBytes + kMergeBytes + kPBytes + 2 * kStages * 8 + 16 +
+        return (size_t)kStagesBytes + kBarBytes + kPBytes + kMergeBytes + 16 +
                (size_t)(B + 1) * 8;
     }
 };
-
-__device__ __forceinline__ void consumer_sync(int nthreads) {
-    asm volatile("bar.sync 1, %0;" ::"r"(nthreads) : "memory");
-}
 
 // Largest b in [0, B) with H_kv * cum[b] <= u (the request holding unit u).
 __device__ __forceinline__ int find_request(const int64_t *cum, int B, int64_t H_kv, int64_t u) {
@@ -105,23 +119,23 @@ __device__ __forceinline__ int64_t cta_of(int64_t u, int64_t U, int64_t C) {
 }
 
 template <typename T, int D, int G>
-__global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
+__global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, G>::kCtasPerSm)
     decode_attn_kernel(const T *__restrict__ q, const T *__restrict__ kc,
                        const T *__restrict__ vc, const int64_t *__restrict__ cache_off,
                        const int32_t *__restrict__ len_in, T *__restrict__ out, float qscale,
                        int B, int H_kv, float *__restrict__ partials, int slot_floats,
                        int *__restrict__ counters, int *__restrict__ err) {
     using C = DecodeCfg<T, D, G>;
-    constexpr int kConsumers = C::kWarps * 32;
+    constexpr int W = C::kWarps, S = C::kStages, TR = C::kTileRows, RW = C::kRowsPerWarp;
     extern __shared__ __align__(128) unsigned char smem[];
     unsigned char *stages = smem;
-    float *mrg_o = reinterpret_cast<float *>(smem + (size_t)C::kStages * C::kStageBytes);
-    float *mrg_m = mrg_o + C::kWarps * G * D;
-    float *mrg_l = mrg_m + C::kWarps * G;
-    float *pbuf = mrg_l + C::kWarps * G;
-    uint64_t *full_bar = reinterpret_cast<uint64_t *>(pbuf + C::kWarps * C::kRowsPerWarp * G);
-    uint64_t *empty_bar = full_bar + C::kStages;
-    volatile int *flags = reinterpret_cast<volatile int *>(empty_bar + C::kStages);
+    uint64_t *full_bar = reinterpret_cast<uint64_t *>(smem + C::kStagesBytes);  // [S]
+    uint64_t *empty_bar = full_bar + S;                                       // [S]
+    uint64_t *piece_bar = full_bar + 2 * S;  // [2]: the consumers deposited a piece
+    uint64_t *free_bar = piece_bar + 2;      // [2]: the merge warp released a buffer
+    float2 *pbuf = reinterpret_cast<float2 *>(smem + C::kStagesBytes + C::kBarBytes);
+    float *mrg = reinterpret_cast<float *>(pbuf + W * RW * G);  // [2][kMergeFloats]
+    volatile int *flags = reinterpret_cast<volatile int *>(mrg + 2 * C::kMergeFloats);
     int64_t *cum = reinterpret_cast<int64_t *>(const_cast<int *>(flags) + 4);
 
     const int tid = threadIdx.x;
@@ -144,11 +158,13 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
     if (tid == 0) {
         cum[0] = 0;
         flags[0] = 0;  // abort
-        flags[1] = 0;  // "this CTA merges" ticket result
-        flags[2] = 0;  // abort flag as seen by all consumers at a piece's end
-        for (int s = 0; s < C::kStages; s++) {
+        for (int s = 0; s < S; s++) {
             mbar_init(&full_bar[s], 1);
-            mbar_init(&empty_bar[s], C::kWarps);
+            mbar_init(&empty_bar[s], W);
+        }
+        for (int x = 0; x < 2; x++) {
+            mbar_init(&piece_bar[x], W);
+            mbar_init(&free_bar[x], 1);
         }
         fence_mbar_init();
     }
@@ -183,7 +199,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
     if (c >= Cn) return;
     const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
 
-    if (warp == C::kWarps) {
+    if (warp == W) {
         // ================= producer: one lane issues bulk copies ============
         if (lane != 0) return;
         int stage = 0;
@@ -194,7 +210,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
             const Piece p = piece_at(cum, B, H_kv, u, u1);
             const int64_t cap = cache_off[p.b + 1] - cache_off[p.b];
             const int64_t base = cache_off[p.b] * H_kv + (int64_t)p.h * cap;
-            for (int64_t t = p.t0; t < p.t1; t += C::kTileRows) {
+            for (int64_t t = p.t0; t < p.t1; t += TR) {
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
                 if (flags[0] || !mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, err) ||
@@ -203,14 +219,18 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
                     stop = true;
                     break;
                 }
-                const int rows = (int)((p.t1 - t) < C::kTileRows ? (p.t1 - t) : C::kTileRows);
+                const int rows = (int)((p.t1 - t) < TR ? (p.t1 - t) : TR);
                 const uint32_t bytes = (uint32_t)rows * C::kRowBytes;
+                const bool first = (t == p.t0);
                 unsigned char *dst = stages + (size_t)stage * C::kStageBytes;
-                mbar_arrive_expect_tx(&full_bar[stage], 2 * bytes);
+                mbar_arrive_expect_tx(&full_bar[stage], 2 * bytes + (first ? C::kQBytes : 0));
                 bulk_g2s(dst, kc + (base + t) * D, bytes, &full_bar[stage]);
                 bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, bytes, &full_bar[stage]);
+                if (first)
+                    bulk_g2s(dst + 2 * C::kTileBytes, q + ((int64_t)p.b * H_q + p.h * G) * D,
+                             C::kQBytes, &full_bar[stage]);
                 ++issued;
-                if (++stage == C::kStages) {
+                if (++stage == S) {
                     stage = 0;
                     phase ^= 1u;
                 }
@@ -218,212 +238,313 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, 1)
             u += p.t1 - p.t0;
         }
         // Let the copies still in flight land before the CTA may exit.
-        const int64_t first = issued > C::kStages ? issued - C::kStages : 0;
+        const int64_t first = issued > S ? issued - S : 0;
         for (int64_t k = first; k < issued; k++)
-            if (!mbar_wait_bounded(&full_bar[k % C::kStages], (uint32_t)((k / C::kStages) & 1), err))
-                break;
+            if (!mbar_wait_bounded(&full_bar[k % S], (uint32_t)((k / S) & 1), err)) break;
         return;
     }
 
-    // ===================== consumers: 8 warps ==============================
-    const int lrow = lane >> 2;  // row of the lane's group within 8 rows
-    const int lq = lane & 3;     // quarter of the row the lane reads
-    const int ctid = tid;        // 0 .. kConsumers-1
+    if (warp == W + 1) {
+        // ======== merge warp: combines the consumers' states of each piece ====
+        // lane owns kCols consecutive output columns of every query head
+        constexpr int kCols = D / 32;
+        constexpr int kBatch = 8;  // partials fetched per round of the final merge
+        int64_t k = 0;             // piece index within this CTA
+        for (int64_t u = u0; u < u1; k++) {
+            const Piece p = piece_at(cum, B, H_kv, u, u1);
+            const int x = (int)(k & 1);
+            const uint32_t use = (uint32_t)((k >> 1) & 1);
+            bool ok = !flags[0] && mbar_wait_bounded(&piece_bar[x], use, err);
+            ok = __all_sync(0xffffffffu, ok) && !__shfl_sync(0xffffffffu, flags[0], 0);
+            const float *mo = mrg + x * C::kMergeFloats;  // [W][G][D]
+            const float *mm = mo + W * G * D;              // [W][G]
+            const float *ml = mm + W * G;                  // [W][G]
+            const int64_t seg = (int64_t)p.b * H_kv + p.h;
+            const bool whole = (p.t0 == 0 && p.t1 == p.L);
+            float *slot = partials + (c + seg) * slot_floats;  // o [G][D], m [G], l [G]
+            if (ok) {
+#pragma unroll
+                for (int g = 0; g < G; g++) {
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int w = 0; w < W; w++) M = fmaxf(M, mm[w * G + g]);
+                    float Ls = 0.f, acc[kCols];
+#pragma unroll
+                    for (int i = 0; i < kCols; i++) acc[i] = 0.f;
+#pragma unroll
+                    for (int w = 0; w < W; w++) {
+                        const float sc = fast_exp2(mm[w * G + g] - M);  // idle warp: 0
+                        Ls = fmaf(ml[w * G + g], sc, Ls);
+                        const float *src = mo + (w * G + g) * D + lane * kCols;
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) acc[i] = fmaf(src[i], sc, acc[i]);
+                    }
+                    if (whole) {
+                        const float inv = 1.f / Ls;
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) acc[i] *= inv;
+                        store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
+                                                lane * kCols,
+                                            acc);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) slot[g * D + lane * kCols + i] = acc[i];
+                        if (lane == 0) {
+                            slot[G * D + g] = M;
+                            slot[G * D + G + g] = Ls;
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&free_bar[x]);  // the buffer may be refilled
+            if (ok && !whole) {
+                // the last CTA to finish a piece of this (request, head) merges
+                // all of its pieces (publish this CTA's partial first)
+                const int64_t A = (int64_t)H_kv * cum[p.b] + (int64_t)p.h * p.L;
+                const int64_t cfirst = cta_of(A, U, Cn), clast = cta_of(A + p.L - 1, U, Cn);
+                int last = 0;
+                if (lane == 0)
+                    last = atomic_add_acq_rel_gpu(&counters[seg], 1) == (int)(clast - cfirst);
+                last = __shfl_sync(0xffffffffu, last, 0);
+                __syncwarp();  // lane 0's acquire orders the other lanes' reads too
+                if (last) {
+#pragma unroll 1
+                    for (int g = 0; g < G; g++) {
+                        // online log-sum-exp over the pieces, kBatch loads in flight
+                        float M = -INFINITY, Ls = 0.f, acc[kCols];
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) acc[i] = 0.f;
+#pragma unroll 1
+                        for (int64_t c0 = cfirst; c0 <= clast; c0 += kBatch) {
+                            float bm[kBatch], bl[kBatch], bo[kBatch][kCols];
+#pragma unroll
+                            for (int j = 0; j < kBatch; j++) {
+                                bm[j] = -INFINITY;
+                                bl[j] = 0.f;
+#pragma unroll
+                                for (int i = 0; i < kCols; i++) bo[j][i] = 0.f;
+                                if (c0 + j <= clast) {
+                                    const float *sp = partials + (c0 + j + seg) * slot_floats;
+                                    bm[j] = __ldcg(sp + G * D + g);
+                                    bl[j] = __ldcg(sp + G * D + G + g);
+#pragma unroll
+                                    for (int i = 0; i < kCols; i++)
+                                        bo[j][i] = __ldcg(sp + g * D + lane * kCols + i);
+                                }
+                            }
+                            float Mn = M;
+#pragma unroll
+                            for (int j = 0; j < kBatch; j++) Mn = fmaxf(Mn, bm[j]);
+                            const float r = fast_exp2(M - Mn);  // 0 while M = -inf
+                            Ls *= r;
+#pragma unroll
+                            for (int i = 0; i < kCols; i++) acc[i] *= r;
+#pragma unroll
+                            for (int j = 0; j < kBatch; j++) {
+                                const float sc = fast_exp2(bm[j] - Mn);  // absent: 0
+                                Ls = fmaf(bl[j], sc, Ls);
+#pragma unroll
+                                for (int i = 0; i < kCols; i++) acc[i] = fmaf(bo[j][i], sc, acc[i]);
+                            }
+                            M = Mn;
+                        }
+                        const float inv = 1.f / Ls;
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) acc[i] *= inv;
+                        store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
+                                                lane * kCols,
+                                            acc);
+                    }
+                    if (lane == 0) counters[seg] = 0;
+                }
+            }
+            u += p.t1 - p.t0;
+        }
+        return;
+    }
+
+    // ===================== consumers: W warps ==============================
+    const int lrow = lane >> 2;  // row within an 8-row pass
+    const int lq = lane & 3;     // quarter of the row
     int ch[C::kChunksPerLane];   // the lane's chunks, rotated by row parity
 #pragma unroll
     for (int i = 0; i < C::kChunksPerLane; i++)
         ch[i] = lq + 4 * ((i + (lrow & 1)) % C::kChunksPerLane);
-    float *pw = pbuf + warp * C::kRowsPerWarp * G;
+    const int pc = lane % C::kPvLanesPerRow;  // PV: 16-byte column chunk
+    const int pr = lane / C::kPvLanesPerRow;  // PV: row within a pass
+    float2 *pw = pbuf + warp * RW * G;
+    const float2 qs = make_float2(qscale, qscale);
 
     int stage = 0;
     uint32_t phase = 0;
     bool aborted = false;
-    for (int64_t u = u0; u < u1;) {
+    int64_t k = 0;  // piece index within this CTA
+    for (int64_t u = u0; u < u1; k++) {
         const Piece p = piece_at(cum, B, H_kv, u, u1);
-        const int b = p.b, h = p.h;
 
-        // query fragments of the group's G heads, pre-scaled by log2(e)/sqrt(d)
-        float qf[G][C::kChunksPerLane][C::kElemsPerChunk];
-#pragma unroll
-        for (int g = 0; g < G; g++)
-#pragma unroll
-            for (int i = 0; i < C::kChunksPerLane; i++) {
-                load_vec<T, C::kElemsPerChunk>(
-                    q + ((int64_t)b * H_q + h * G + g) * D + ch[i] * C::kElemsPerChunk, qf[g][i]);
-#pragma unroll
-                for (int e = 0; e < C::kElemsPerChunk; e++) qf[g][i][e] *= qscale;
-            }
-        float m[G], l[G], o[G][C::kColsPerLane];
+        float2 q2[G][C::kChunksPerLane][C::kPairsPerChunk];
+        float m[G], l[G];
+        float2 o[G][C::kPairsPerChunk];
 #pragma unroll
         for (int g = 0; g < G; g++) {
             m[g] = -INFINITY;
             l[g] = 0.f;
 #pragma unroll
-            for (int cc = 0; cc < C::kColsPerLane; cc++) o[g][cc] = 0.f;
+            for (int e = 0; e < C::kPairsPerChunk; e++) o[g][e] = make_float2(0.f, 0.f);
         }
 
-        for (int64_t t = p.t0; t < p.t1; t += C::kTileRows) {
-            const int rows = (int)((p.t1 - t) < C::kTileRows ? (p.t1 - t) : C::kTileRows);
-            if (!aborted && (flags[0] || !mbar_wait_bounded(&full_bar[stage], phase, err))) {
-                flags[0] = 1;
-                aborted = true;
+        for (int64_t t = p.t0; t < p.t1; t += TR) {
+            const int rows = (int)((p.t1 - t) < TR ? (p.t1 - t) : TR);
+            if (!aborted) {
+                // warp-uniform decision: every lane waits, any failure stops the warp
+                bool fail = flags[0] != 0;
+                if (!fail) fail = !mbar_wait_bounded(&full_bar[stage], phase, err);
+                if (__any_sync(0xffffffffu, fail)) {
+                    flags[0] = 1;
+                    aborted = true;
+                }
             }
             const unsigned char *ks = stages + (size_t)stage * C::kStageBytes;
-            const unsigned char *vs = ks + C::kTileBytes;
-            const int r0 = warp * C::kRowsPerWarp;
-            int nw = rows - r0;
-            nw = nw < 0 ? 0 : (nw > C::kRowsPerWarp ? C::kRowsPerWarp : nw);
-            if (nw > 0 && !aborted) {
-                // ---- scores s = (q * log2e/sqrt(d)) . k for the warp's rows
-                float s[G][C::kRowsPerGroup];
+            if (!aborted && t == p.t0) {
+                // the piece's queries came with its first tile; scale them by
+                // log2(e)/sqrt(d) so that scores are in base 2
 #pragma unroll
-                for (int rr = 0; rr < C::kRowsPerGroup; rr++) {
-                    const int row = r0 + rr * 8 + lrow;
-                    const unsigned char *kr = ks + row * C::kRowBytes;
-                    float acc[G][2];
-#pragma unroll
-                    for (int g = 0; g < G; g++) acc[g][0] = acc[g][1] = 0.f;
+                for (int g = 0; g < G; g++)
 #pragma unroll
                     for (int i = 0; i < C::kChunksPerLane; i++) {
-                        float kf[C::kElemsPerChunk];
-                        load_vec<T, C::kElemsPerChunk>(reinterpret_cast<const T *>(kr + ch[i] * 16), kf);
+                        load16_pairs<T>(ks + 2 * C::kTileBytes + g * C::kRowBytes + ch[i] * 16,
+                                        q2[g][i]);
 #pragma unroll
-                        for (int e = 0; e < C::kElemsPerChunk; e++)
+                        for (int e = 0; e < C::kPairsPerChunk; e++)
+                            q2[g][i][e] = fmul2(q2[g][i][e], qs);
+                    }
+            }
+            const unsigned char *vs = ks + C::kTileBytes;
+            const int r0 = warp * RW;
+            int nw = rows - r0;
+            nw = nw < 0 ? 0 : (nw > RW ? RW : nw);
+            if (nw > 0 && !aborted) {
+                // ---- scores (q * log2e/sqrt(d)) . k, two packed partial sums
+                float s[G][C::kQkPasses];
 #pragma unroll
-                            for (int g = 0; g < G; g++)
-                                acc[g][e & 1] = fmaf(qf[g][i][e], kf[e], acc[g][e & 1]);
+                for (int rr = 0; rr < C::kQkPasses; rr++) {
+                    const int row = rr * 8 + lrow;
+                    const unsigned char *kr = ks + (r0 + row) * C::kRowBytes;
+                    float2 acc[G];
+#pragma unroll
+                    for (int g = 0; g < G; g++) acc[g] = make_float2(0.f, 0.f);
+#pragma unroll
+                    for (int i = 0; i < C::kChunksPerLane; i++) {
+                        float2 k2[C::kPairsPerChunk];
+                        load16_pairs<T>(kr + ch[i] * 16, k2);
+#pragma unroll
+                        for (int e = 0; e < C::kPairsPerChunk; e++)
+#pragma unroll
+                            for (int g = 0; g < G; g++) acc[g] = ffma2(q2[g][i][e], k2[e], acc[g]);
                     }
 #pragma unroll
                     for (int g = 0; g < G; g++) {
-                        float v = acc[g][0] + acc[g][1];
+                        float v = acc[g].x + acc[g].y;
                         v += __shfl_xor_sync(0xffffffffu, v, 1);
                         v += __shfl_xor_sync(0xffffffffu, v, 2);
-                        s[g][rr] = (row < rows) ? v : -INFINITY;
+                        s[g][rr] = (row < nw) ? v : -INFINITY;
                     }
                 }
-                // ---- online softmax update (warp-wide running max)
+                // ---- online softmax update (warp-wide running max and sum)
 #pragma unroll
                 for (int g = 0; g < G; g++) {
                     float mt = s[g][0];
 #pragma unroll
-                    for (int rr = 1; rr < C::kRowsPerGroup; rr++) mt = fmaxf(mt, s[g][rr]);
+                    for (int rr = 1; rr < C::kQkPasses; rr++) mt = fmaxf(mt, s[g][rr]);
                     mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 4));
                     mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 8));
                     mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, 16));
                     const float mnew = fmaxf(m[g], mt);
                     const float corr = fast_exp2(m[g] - mnew);
                     m[g] = mnew;
-                    l[g] *= corr;
+                    float ps = 0.f;
 #pragma unroll
-                    for (int cc = 0; cc < C::kColsPerLane; cc++) o[g][cc] *= corr;
-#pragma unroll
-                    for (int rr = 0; rr < C::kRowsPerGroup; rr++) {
-                        const float pr = fast_exp2(s[g][rr] - mnew);
-                        if (lq == 0) pw[(rr * 8 + lrow) * G + g] = pr;
+                    for (int rr = 0; rr < C::kQkPasses; rr++) {
+                        const float pv = fast_exp2(s[g][rr] - mnew);
+                        ps += pv;
+                        if (lq == 0) pw[(rr * 8 + lrow) * G + g] = make_float2(pv, pv);
                     }
+                    ps += __shfl_xor_sync(0xffffffffu, ps, 4);
+                    ps += __shfl_xor_sync(0xffffffffu, ps, 8);
+                    ps += __shfl_xor_sync(0xffffffffu, ps, 16);
+                    l[g] = fmaf(l[g], corr, ps);
+                    const float2 c2 = make_float2(corr, corr);
+#pragma unroll
+                    for (int e = 0; e < C::kPairsPerChunk; e++) o[g][e] = fmul2(o[g][e], c2);
                 }
                 __syncwarp();
                 // ---- o += p * v over the warp's valid rows
-                const T *vrow = reinterpret_cast<const T *>(vs + r0 * C::kRowBytes) +
-                                lane * C::kColsPerLane;
+                const unsigned char *vw = vs + r0 * C::kRowBytes + pc * 16;
 #pragma unroll 4
-                for (int j = 0; j < nw; j++) {
-                    float vf[C::kColsPerLane];
-                    load_vec<T, C::kColsPerLane>(vrow + j * D, vf);
+                for (int j0 = 0; j0 < nw; j0 += C::kPvRowsPerPass) {
+                    const int row = j0 + pr;
+                    if (row < nw) {
+                        float2 v2[C::kPairsPerChunk];
+                        load16_pairs<T>(vw + row * C::kRowBytes, v2);
 #pragma unroll
-                    for (int g = 0; g < G; g++) {
-                        const float pj = pw[j * G + g];
-                        l[g] += pj;
+                        for (int g = 0; g < G; g++) {
+                            const float2 pg = pw[row * G + g];
 #pragma unroll
-                        for (int cc = 0; cc < C::kColsPerLane; cc++)
-                            o[g][cc] = fmaf(pj, vf[cc], o[g][cc]);
+                            for (int e = 0; e < C::kPairsPerChunk; e++)
+                                o[g][e] = ffma2(pg, v2[e], o[g][e]);
+                        }
                     }
                 }
-                __syncwarp();
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty_bar[stage]);
-            if (++stage == C::kStages) {
+            if (++stage == S) {
                 stage = 0;
                 phase ^= 1u;
             }
         }
 
-        // ---- merge the 8 warps' states of this piece
+        // ---- deposit this warp's state of the piece for the merge warp
+        // (fold the PV row groups onto lanes with pr == 0 first)
 #pragma unroll
-        for (int g = 0; g < G; g++) {
+        for (int g = 0; g < G; g++)
 #pragma unroll
-            for (int cc = 0; cc < C::kColsPerLane; cc++)
-                mrg_o[(warp * G + g) * D + lane * C::kColsPerLane + cc] = o[g][cc];
-            if (lane == 0) {
-                mrg_m[warp * G + g] = m[g];
-                mrg_l[warp * G + g] = l[g];
+            for (int e = 0; e < C::kPairsPerChunk; e++)
+#pragma unroll
+                for (int off = C::kPvLanesPerRow; off < 32; off <<= 1) {
+                    o[g][e].x += __shfl_xor_sync(0xffffffffu, o[g][e].x, off);
+                    o[g][e].y += __shfl_xor_sync(0xffffffffu, o[g][e].y, off);
+                }
+        const int x = (int)(k & 1);
+        // buffer x was last used by piece k - 2: wait until the merge warp
+        // released it (the first use of each buffer passes at once)
+        if (!aborted) {
+            bool fail = !mbar_wait_bounded(&free_bar[x], (uint32_t)(((k >> 1) & 1) ^ 1), err);
+            if (__any_sync(0xffffffffu, fail)) {
+                flags[0] = 1;
+                aborted = true;
             }
         }
-        consumer_sync(kConsumers);
-        if (ctid == 0) flags[2] = flags[0];
-        consumer_sync(kConsumers);
-        // uniform over the consumers (all branches below that hold a barrier
-        // depend only on values every consumer warp agrees on)
-        const bool stop = flags[2] != 0;
-        const bool whole = (p.t0 == 0 && p.t1 == p.L);
-        const int64_t seg = (int64_t)b * H_kv + h;
-        if (!stop) {
-            for (int idx = ctid; idx < G * D; idx += kConsumers) {
-                const int g = idx / D, col = idx - g * D;
-                float M = -INFINITY;
+        float *mo = mrg + x * C::kMergeFloats;
+        if (pr == 0) {
 #pragma unroll
-                for (int w = 0; w < C::kWarps; w++) M = fmaxf(M, mrg_m[w * G + g]);
-                float Ls = 0.f, O = 0.f;
+            for (int g = 0; g < G; g++)
 #pragma unroll
-                for (int w = 0; w < C::kWarps; w++) {
-                    const float sc = fast_exp2(mrg_m[w * G + g] - M);
-                    Ls = fmaf(mrg_l[w * G + g], sc, Ls);
-                    O = fmaf(mrg_o[(w * G + g) * D + col], sc, O);
+                for (int e = 0; e < C::kPairsPerChunk; e++) {
+                    const int col = pc * (16 / (int)sizeof(T)) + 2 * e;
+                    *reinterpret_cast<float2 *>(&mo[(warp * G + g) * D + col]) = o[g][e];
                 }
-                if (whole) {
-                    out[((int64_t)b * H_q + h * G + g) * D + col] = from_float<T>(O / Ls);
-                } else {
-                    float *slot = partials + (c + seg) * slot_floats;
-                    slot[2 * G + g * D + col] = O;
-                    if (col == 0) {
-                        slot[g] = M;
-                        slot[G + g] = Ls;
-                    }
-                }
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int g = 0; g < G; g++) {
+                mo[W * G * D + warp * G + g] = m[g];
+                mo[W * G * D + W * G + warp * G + g] = l[g];
             }
         }
-        if (!whole && !stop) {
-            // ---- last-arriving CTA of this (request, head) merges the pieces
-            __threadfence();
-            consumer_sync(kConsumers);
-            const int64_t A = (int64_t)H_kv * cum[b] + (int64_t)h * p.L;
-            const int64_t cfirst = cta_of(A, U, Cn), clast = cta_of(A + p.L - 1, U, Cn);
-            if (ctid == 0) {
-                const int old = atomicAdd(&counters[seg], 1);
-                flags[1] = (old == (int)(clast - cfirst));
-            }
-            consumer_sync(kConsumers);
-            if (flags[1]) {
-                __threadfence();
-                for (int idx = ctid; idx < G * D; idx += kConsumers) {
-                    const int g = idx / D, col = idx - g * D;
-                    float M = -INFINITY;
-                    for (int64_t cp = cfirst; cp <= clast; cp++)
-                        M = fmaxf(M, __ldcg(partials + (cp + seg) * slot_floats + g));
-                    float Ls = 0.f, O = 0.f;
-                    for (int64_t cp = cfirst; cp <= clast; cp++) {
-                        const float *slot = partials + (cp + seg) * slot_floats;
-                        const float sc = fast_exp2(__ldcg(slot + g) - M);
-                        Ls = fmaf(__ldcg(slot + G + g), sc, Ls);
-                        O = fmaf(__ldcg(slot + 2 * G + g * D + col), sc, O);
-                    }
-                    out[((int64_t)b * H_q + h * G + g) * D + col] = from_float<T>(O / Ls);
-                }
-                if (ctid == 0) counters[seg] = 0;
-            }
-        }
-        consumer_sync(kConsumers);  // merge buffers are reused by the next piece
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&piece_bar[x]);
         u += p.t1 - p.t0;
     }
 }
@@ -436,15 +557,17 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev < 31 && !(__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev))) {
+    const bool cached =
+        dev < 31 && (__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev));
+    if (!cached) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)C::smem_bytes(SPEECHKV_MAX_BATCH));
         if (e != cudaSuccess) return e;
-        __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
-    } else if (dev >= 31) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)C::smem_bytes(SPEECHKV_MAX_BATCH));
+        // all of the unified L1/shared storage as shared memory, so that
+        // kCtasPerSm CTAs fit on an SM
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
+        if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
     }
     const float qscale = a.scale * 1.4426950408889634f;  // log2(e): scores in base 2
     kern<<<grid, C::kThreads, C::smem_bytes(a.B), stream>>>(
@@ -454,16 +577,19 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
     return cudaGetLastError();
 }
 
+// Resident CTAs per SM for a batch of B requests (the length table in shared
+// memory grows with B).
 template <typename T, int D, int G>
-int occupancy_instance() {
+int occupancy_instance(int B) {
     using C = DecodeCfg<T, D, G>;
     auto kern = decode_attn_kernel<T, D, G>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)C::smem_bytes(SPEECHKV_MAX_BATCH)) != cudaSuccess)
+                             (int)C::smem_bytes(SPEECHKV_MAX_BATCH)) != cudaSuccess ||
+        cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100) !=
+            cudaSuccess)
         return 0;
     int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, C::kThreads,
-                                                      C::smem_bytes(SPEECHKV_MAX_BATCH)) !=
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, C::kThreads, C::smem_bytes(B)) !=
         cudaSuccess)
         return 0;
     return n;
@@ -481,9 +607,9 @@ int decode_slot_floats(int d, int group) {
     return (f + 3) & ~3;  // keep slots 16-byte aligned
 }
 
-#define SPEECHKV_DECODE_CASES(X)                                          \
-    X(float, 64, 1) X(float, 64, 2) X(float, 64, 4)                       \
-    X(float, 128, 1) X(float, 128, 2) X(float, 128, 4)                    \
+#define SPEECHKV_DECODE_CASES(X)                                            \
+    X(float, 64, 1) X(float, 64, 2) X(float, 64, 4)                         \
+    X(float, 128, 1) X(float, 128, 2) X(float, 128, 4)                      \
     X(__nv_bfloat16, 64, 1) X(__nv_bfloat16, 64, 2) X(__nv_bfloat16, 64, 4) \
     X(__nv_bfloat16, 128, 1) X(__nv_bfloat16, 128, 2) X(__nv_bfloat16, 128, 4)
 
@@ -492,9 +618,9 @@ constexpr speechkv_dtype dtype_of() {
     return sizeof(T) == 4 ? SPEECHKV_F32 : SPEECHKV_BF16;
 }
 
-int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group) {
+int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B) {
 #define X(T, D, G) \
-    if (dtype == dtype_of<T>() && d == D && group == G) return occupancy_instance<T, D, G>();
+    if (dtype == dtype_of<T>() && d == D && group == G) return occupancy_instance<T, D, G>(B);
     SPEECHKV_DECODE_CASES(X)
 #undef X
     return 0;
@@ -502,8 +628,9 @@ int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group) {
 
 cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream) {
     const int group = a.H_q / a.H_kv;
-#define X(T, D, G) \
-    if (a.dtype == dtype_of<T>() && a.d == D && group == G) return launch_instance<T, D, G>(a, grid, stream);
+#define X(T, D, G)                                                  \
+    if (a.dtype == dtype_of<T>() && a.d == D && group == G)         \
+        return launch_instance<T, D, G>(a, grid, stream);
     SPEECHKV_DECODE_CASES(X)
 #undef X
     return cudaErrorInvalidValue;

@@ -51,8 +51,9 @@ struct DecodeArgs {
 
 // Whether (dtype, d, group) has a compiled decode kernel.
 bool decode_supported(speechkv_dtype dtype, int d, int group);
-// Resident CTAs per SM of that kernel on the current device (0 on error).
-int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group);
+// Resident CTAs per SM of that kernel on the current device for a batch of
+// B requests (0 on error).
+int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B);
 // Floats per partial-result slot (m, l and o for every query head of a group).
 int decode_slot_floats(int d, int group);
 cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream);

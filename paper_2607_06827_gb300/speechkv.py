@@ -18,7 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libspeechkv.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_CAPACITY, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
 F32, BF16 = 0, 1
-MAX_BATCH = 2048
+MAX_BATCH = 1024
 
 # Every function the header declares: name -> (restype, argtypes)
 _P = ctypes.c_void_p
