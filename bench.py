@@ -65,6 +65,8 @@ def parse_args():
     ap.add_argument("--no-sweep", action="store_true")
     ap.add_argument("--no-w1", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-unfused", action="store_true",
+                    help="skip timing append + decode_attn as two launches")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="budget of the oracle CPU baseline sample")
@@ -231,24 +233,34 @@ class DecodeModel:
         status = sk.check_device_error()
         assert status == sk.OK, sk.status_string(status)
 
-    def launch_step(self, s: int, events=None):
+    def launch_step(self, s: int, events=None, fused: bool = True):
+        """One decode step over all layers: speechkv_decode_step (append fused
+        into the attention launch), or speechkv_append + speechkv_decode_attn."""
         wl, sk = self.wl, self.sk
         for i, layer in enumerate(self.layers):
-            sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
-                      self.len[i], wl.w, layer, wl.l0)
+            if not fused:
+                sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
+                          self.len[i], wl.w, layer, wl.l0)
             if events is not None:
                 events[i][0].record()
-            sk.decode_attn(self.q[s, i], self.k[i], self.v[i], self.off[i], self.len[i],
-                           self.out[i], self.ws, wl.w, layer, wl.l0, wl.H_kv)
+            if fused:
+                sk.decode_step(self.q[s, i], self.kn[s, i], self.vn[s, i], self.k[i], self.v[i],
+                               self.off[i], self.len[i], self.out[i], self.ws, wl.w, layer,
+                               wl.l0)
+            else:
+                sk.decode_attn(self.q[s, i], self.k[i], self.v[i], self.off[i], self.len[i],
+                               self.out[i], self.ws, wl.w, layer, wl.l0, wl.H_kv)
             if events is not None:
                 events[i][1].record()
 
-    def attn_bytes(self, rows_per_req) -> int:
-        """Algorithmic bytes of one decode_attn launch: every cached K and V
-        row once, the queries and the outputs (bf16)."""
+    def attn_bytes(self, rows_per_req, fused: bool = True) -> int:
+        """Algorithmic bytes of one decode-attention launch: every K and V row
+        attended to once (the new token's included), the queries and the
+        outputs; the fused step also writes the new token's row (bf16)."""
         wl = self.wl
         kv = sum(rows_per_req) * wl.H_kv * wl.d * 2 * 2
-        return kv + 2 * wl.B * wl.H_q * wl.d * 2
+        new_rows = wl.B * wl.H_kv * wl.d * 2 * 2 if fused else 0
+        return kv + 2 * wl.B * wl.H_q * wl.d * 2 + new_rows
 
     def free(self):
         for name in ("k", "v", "len", "off", "q", "kn", "vn", "out", "ws"):
@@ -256,7 +268,7 @@ class DecodeModel:
 
 
 def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist: Dist,
-              clocks: ClockSampler | None, kernel_events: bool = True):
+              clocks: ClockSampler | None, kernel_events: bool = True, fused: bool = True):
     """Capture `steps` decode steps in CUDA graphs of `chunk` steps, then replay
     them as the timed region.  Returns (region_ms, per-layer attn ms lists)."""
     import torch
@@ -270,7 +282,7 @@ def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
             for i in range(n):
-                model.launch_step(s + i, ev[i] if ev else None)
+                model.launch_step(s + i, ev[i] if ev else None, fused=fused)
         graphs.append(g)
         evs.append(ev)
         s += n
@@ -298,19 +310,25 @@ def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist:
 
 
 def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int,
-            layers=None):
-    """Build the model for `wl`, run warm-up steps eagerly, time `steps`
-    graph-replayed steps.  Returns a result dict."""
+            layers=None, fused: bool = True):
+    """Build the model for `wl`, run warm-up steps eagerly, then two timed
+    passes of `steps` graph-replayed decode steps each: the first with no
+    events inside the graphs (the step time), the second with CUDA events
+    around every decode-attention launch (per-kernel durations for the
+    roofline).  Returns a result dict."""
     import torch
-    model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key, layers=layers)
+    model = DecodeModel(wl, steps_total=warmup + 2 * steps, seed_key=seed_key, layers=layers)
     for s in range(warmup):
-        model.launch_step(s)
+        model.launch_step(s, fused=fused)
     torch.cuda.synchronize()
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
     L = len(model.layers)
-    base_rows = [[model.rows0[i][b] + warmup for b in range(wl.B)] for i in range(L)]
-    region_ms, per_layer = run_timed(model, warmup, steps, chunk, dist, clocks)
+    region_ms, _ = run_timed(model, warmup, steps, chunk, dist, clocks, kernel_events=False,
+                             fused=fused)
+    base_rows = [[model.rows0[i][b] + warmup + steps for b in range(wl.B)] for i in range(L)]
+    events_region_ms, per_layer = run_timed(model, warmup + steps, steps, chunk, dist, clocks,
+                                            kernel_events=True, fused=fused)
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
     comp = [i for i, layer in enumerate(model.layers) if layer >= wl.l0]
@@ -319,7 +337,7 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
     ratio = lambda a, b: a / b if b else float("nan")  # noqa: E731
     attn_ms = {i: mean(per_layer[i]) for i in range(L)}
     # algorithmic bytes: rows after step t's append are base + t + 1
-    bytes_total = {i: sum(model.attn_bytes([r + t + 1 for r in base_rows[i]])
+    bytes_total = {i: sum(model.attn_bytes([r + t + 1 for r in base_rows[i]], fused)
                           for t in range(steps)) for i in range(L)}
     time_total = {i: sum(per_layer[i]) for i in range(L)}
     res = {
@@ -338,8 +356,11 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
         "attn_bytes_per_launch_all": sum(bytes_total.values()) / (L * steps),
         "pool_us_compressed_layer": mean([model.pool_ms[model.layers[i]] for i in comp]) * 1e3,
         "pool_us_full_layer": mean([model.pool_ms[model.layers[i]] for i in full]) * 1e3,
-        "gpu_launches": steps * L * 2,
+        "gpu_launches": steps * L * (1 if fused else 2),
         "region_ms": region_ms,
+        "events_pass_step_us": events_region_ms * 1e3 / steps,
+        "path": "speechkv_decode_step (append fused)" if fused else
+                "speechkv_append + speechkv_decode_attn",
     }
     model.free()
     del model
@@ -369,10 +390,8 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
             d_q[i].copy_(h_q[s, i], non_blocking=True)
             d_kn[i].copy_(h_kn[s, i], non_blocking=True)
             d_vn[i].copy_(h_vn[s, i], non_blocking=True)
-            sk.append(d_kn[i], d_vn[i], model.k[i], model.v[i], model.off[i], model.len[i],
-                      wl.w, layer, wl.l0)
-            sk.decode_attn(d_q[i], model.k[i], model.v[i], model.off[i], model.len[i],
-                           model.out[i], model.ws, wl.w, layer, wl.l0, Hk)
+            sk.decode_step(d_q[i], d_kn[i], d_vn[i], model.k[i], model.v[i], model.off[i],
+                           model.len[i], model.out[i], model.ws, wl.w, layer, wl.l0)
             h_out[s, i].copy_(model.out[i], non_blocking=True)
 
     for s in range(warmup):
@@ -591,6 +610,10 @@ def main():
         wl1 = inputs.qwen_long_audio(args.minutes, 1, generated=GENERATED)
         w1_res = measure(wl1, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0,
                          layers=layers)
+    unfused = None
+    if not args.no_unfused:
+        unfused = measure(wl, args.sweep_steps, args.warmup, args.graph_chunk, dist, clocks,
+                          seed_key=0, layers=layers, fused=False)
     e2e = None
     if not args.no_e2e:
         e2e = measure_e2e(wl, min(args.e2e_steps, args.steps), args.warmup, args.graph_chunk,
@@ -651,7 +674,8 @@ def main():
                 "bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "peak_kind": peak_kind,
                 "traffic": profiled_traffic(main_res["attn_bytes_per_launch_all"]),
-                "kernel": "speechkv decode_attn (bf16, d=128, group 2), all 28 layers",
+                "kernel": ("decode_attn_kernel (fused append, bf16, d=128, group 2) of "
+                           "speechkv_decode_step, all 28 layers"),
                 "algorithmic_bytes_per_launch": round(main_res["attn_bytes_per_launch_all"]),
                 "compressed_layers": {
                     "achieved": round(main_res["attn_gbs_compressed_layer"], 1),
@@ -669,6 +693,8 @@ def main():
                           for k, v in main_res.items()},
             "w1": ({k: (round(v, 3) if isinstance(v, float) else v) for k, v in w1_res.items()}
                    if w1_res else None),
+            "unfused": ({k: (round(v, 3) if isinstance(v, float) else v)
+                         for k, v in unfused.items()} if unfused else None),
             "speedup_vs_w1": ({
                 "decode_attn_compressed_layer": round(w1_res["attn_us_compressed_layer"] /
                                                       main_res["attn_us_compressed_layer"], 3),

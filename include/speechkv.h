@@ -65,8 +65,8 @@ typedef enum {
 
 typedef enum { SPEECHKV_F32 = 0, SPEECHKV_BF16 = 1 } speechkv_dtype;
 
-/* Largest batch speechkv_decode_attn accepts (its per-CTA length table). */
-#define SPEECHKV_MAX_BATCH 1024
+/* Largest batch speechkv_decode_attn / _step accept (their per-CTA tables). */
+#define SPEECHKV_MAX_BATCH 512
 
 /* Human-readable name of a status (static string, never NULL). */
 const char *speechkv_status_string(speechkv_status status);
@@ -147,8 +147,8 @@ speechkv_status speechkv_append(const void *k_new, const void *v_new,
  * Bytes of workspace speechkv_decode_attn needs for a batch of B requests
  * with the given heads and head dim, launched on `grid_ctas` CTAs (0 = the
  * automatic grid, sized from the current device's SM count).  The workspace
- * holds split-K partial results and one arrival counter per (request, KV
- * head).  Returns 0 for invalid arguments.
+ * holds split-K partial results, one arrival counter per (request, KV head)
+ * and one counter of the fused step.  Returns 0 for invalid arguments.
  */
 size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv,
                                       int32_t d, int32_t grid_ctas);
@@ -194,6 +194,34 @@ speechkv_status speechkv_decode_attn(const void *q, const void *k_cache,
                                      size_t workspace_bytes,
                                      speechkv_dtype dtype,
                                      cudaStream_t stream);
+
+/*
+ * speechkv_decode_step -- one decode step at one layer with the cache update
+ * fused in: speechkv_append followed by speechkv_decode_attn in a single
+ * launch (Sec. III-C: the new token's key/value join the cache uncompressed;
+ * Eq. (attn): the query attends over the cache including that token).
+ *
+ * For every request b with len[b] < cap_b: k_new[b], v_new[b] are written as
+ * cached row len[b] and take part in the attention as that row, and len[b]
+ * advances by one (after every CTA has read it).  A request whose cache is
+ * full sets SPEECHKV_ERR_CAPACITY and attends over its cached rows only.
+ * Results equal speechkv_append then speechkv_decode_attn up to summation
+ * order.
+ *
+ * k_new, v_new   dev, [B][H_kv][d] (16-byte aligned).
+ * All other arguments as for speechkv_decode_attn; len is read and written,
+ * and the caches are written at the new rows.  The workspace (same size as
+ * for speechkv_decode_attn) must not be shared with a concurrent call.
+ */
+speechkv_status speechkv_decode_step(const void *q, const void *k_new,
+                                     const void *v_new, void *k_cache,
+                                     void *v_cache, const int64_t *cache_off,
+                                     int32_t *len, void *out, float scale,
+                                     int32_t B, int32_t H_q, int32_t H_kv,
+                                     int32_t d, int32_t w, int32_t layer,
+                                     int32_t l0, int32_t grid_ctas,
+                                     void *workspace, size_t workspace_bytes,
+                                     speechkv_dtype dtype, cudaStream_t stream);
 
 /*
  * Synchronises `stream`, then reads and clears the current device's error

@@ -98,12 +98,71 @@ speechkv_status decode_auto_grid(DeviceState *s, speechkv_dtype dt, int d, int g
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// Workspace layout: counters [B*H_kv] int32 (256-byte padded), then partial
-// slots [grid + B*H_kv][slot_floats] fp32.
+// Workspace layout: counters [B*H_kv] int32 and one more int32 (the fused
+// step's CTA count), 256-byte padded, then partial slots
+// [grid + B*H_kv][slot_floats] fp32.
+size_t counters_bytes(int B, int H_kv) { return round_up(((size_t)B * H_kv + 1) * 4, 256); }
+
 size_t workspace_bytes(int B, int H_q, int H_kv, int d, int grid) {
     const size_t S = (size_t)B * H_kv;
     const size_t slot = (size_t)speechkv::decode_slot_floats(d, H_q / H_kv);
-    return round_up(S * 4, 256) + ((size_t)grid + S) * slot * 4;
+    return counters_bytes(B, H_kv) + ((size_t)grid + S) * slot * 4;
+}
+
+// Shared by speechkv_decode_attn (k_new == v_new == NULL) and
+// speechkv_decode_step (both non-NULL).
+speechkv_status decode_common(const void *q, const void *k_new, const void *v_new,
+                              void *k_cache, void *v_cache, const int64_t *cache_off,
+                              int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+                              int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+                              int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                              speechkv_dtype dtype, cudaStream_t stream, bool append) {
+    if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
+        grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!q || !k_cache || !v_cache || !cache_off || !len || !out ||
+        (append && (!k_new || !v_new)))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+        !aligned(cache_off, 8) || !aligned(len, 4) ||
+        (append && (!aligned(k_new, 16) || !aligned(v_new, 16))))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    int grid = grid_ctas;
+    if (grid == 0) {
+        st = decode_auto_grid(s, dtype, d, H_q / H_kv, B, &grid);
+        if (st != SPEECHKV_OK) return st;
+    }
+    const size_t need = workspace_bytes(B, H_q, H_kv, d, grid);
+    if (!workspace || workspace_bytes_in < need || !aligned(workspace, 16))
+        return SPEECHKV_ERR_WORKSPACE;
+    speechkv::DecodeArgs a;
+    a.q = q;
+    a.k_new = append ? k_new : nullptr;
+    a.v_new = append ? v_new : nullptr;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.out = out;
+    a.scale = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
+    a.B = B;
+    a.H_q = H_q;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.dtype = dtype;
+    a.counters = static_cast<int *>(workspace);
+    a.done = a.counters + (size_t)B * H_kv;
+    a.partials = reinterpret_cast<float *>(static_cast<char *>(workspace) +
+                                           counters_bytes(B, H_kv));
+    a.err = s->err;
+    return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                   : SPEECHKV_ERR_CUDA;
 }
 
 }  // namespace
@@ -225,47 +284,22 @@ speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const v
                                      int32_t d, int32_t w, int32_t layer, int32_t l0,
                                      int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
                                      speechkv_dtype dtype, cudaStream_t stream) {
-    if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
-        grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale))
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
-    if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
-    if (B == 0) return SPEECHKV_OK;
-    if (!q || !k_cache || !v_cache || !cache_off || !len || !out)
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
-        !aligned(cache_off, 8) || !aligned(len, 4))
-        return SPEECHKV_ERR_INVALID_ARG;
-    DeviceState *s = nullptr;
-    speechkv_status st = device_state(&s);
-    if (st != SPEECHKV_OK) return st;
-    int grid = grid_ctas;
-    if (grid == 0) {
-        st = decode_auto_grid(s, dtype, d, H_q / H_kv, B, &grid);
-        if (st != SPEECHKV_OK) return st;
-    }
-    const size_t need = workspace_bytes(B, H_q, H_kv, d, grid);
-    if (!workspace || workspace_bytes_in < need || !aligned(workspace, 16))
-        return SPEECHKV_ERR_WORKSPACE;
-    speechkv::DecodeArgs a;
-    a.q = q;
-    a.k_cache = k_cache;
-    a.v_cache = v_cache;
-    a.cache_off = cache_off;
-    a.len = len;
-    a.out = out;
-    a.scale = scale > 0.f ? scale : 1.0f / sqrtf((float)d);
-    a.B = B;
-    a.H_q = H_q;
-    a.H_kv = H_kv;
-    a.d = d;
-    a.dtype = dtype;
-    a.counters = static_cast<int *>(workspace);
-    a.partials = reinterpret_cast<float *>(static_cast<char *>(workspace) +
-                                           round_up((size_t)B * H_kv * 4, 256));
-    a.err = s->err;
-    return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
-                                                                   : SPEECHKV_ERR_CUDA;
+    // the caches and len are only read on this path
+    return decode_common(q, nullptr, nullptr, const_cast<void *>(k_cache),
+                         const_cast<void *>(v_cache), cache_off, const_cast<int32_t *>(len), out,
+                         scale, B, H_q, H_kv, d, w, layer, l0, grid_ctas, workspace,
+                         workspace_bytes_in, dtype, stream, false);
+}
+
+speechkv_status speechkv_decode_step(const void *q, const void *k_new, const void *v_new,
+                                     void *k_cache, void *v_cache, const int64_t *cache_off,
+                                     int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+                                     int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                                     speechkv_dtype dtype, cudaStream_t stream) {
+    return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
+                         H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
+                         stream, true);
 }
 
 speechkv_status speechkv_check_device_error(cudaStream_t stream) {

@@ -65,8 +65,12 @@ struct DecodeCfg {
     static constexpr int kMergeBytes = 2 * kMergeFloats * 4;
     static constexpr int kBarBytes = (2 * 3 + 4) * 8;  // full/empty per stage (<= 3), piece/free x2
     static constexpr int kSmemLimit = 227 * 1024;
-    static constexpr int kFixedMax =
-        kBarBytes + kPBytes + kMergeBytes + 16 + (SPEECHKV_MAX_BATCH + 1) * 8;
+    // per-request tables: prefix sums of rows and cache offsets (int64, B+1
+    // each) and the row an appended token takes (int32, B, padded)
+    static size_t table_bytes(int B) { return (size_t)(B + 1) * 16 + ((size_t)B * 4 + 15) / 16 * 16; }
+    static constexpr int kTableMax =
+        (SPEECHKV_MAX_BATCH + 1) * 16 + (SPEECHKV_MAX_BATCH * 4 + 15) / 16 * 16;
+    static constexpr int kFixedMax = kBarBytes + kPBytes + kMergeBytes + 16 + kTableMax;
     static constexpr int kStagesFit = (kSmemLimit - kFixedMax) / kStageBytes;
     static constexpr int kStages = kStagesFit < 3 ? kStagesFit : 3;
     static constexpr int kStagesBytes = kStages * kStageBytes;
@@ -76,8 +80,7 @@ struct DecodeCfg {
     static_assert(kPvLanesPerRow <= 32, "row too long for the PV lane layout");
 
     static size_t smem_bytes(int B) {
-        return (size_t)kStagesBytes + kBarBytes + kPBytes + kMergeBytes + 16 +
-               (size_t)(B + 1) * 8;
+        return (size_t)kStagesBytes + kBarBytes + kPBytes + kMergeBytes + 16 + table_bytes(B);
     }
 };
 
@@ -118,13 +121,17 @@ __device__ __forceinline__ int64_t cta_of(int64_t u, int64_t U, int64_t C) {
     return ((u + 1) * C - 1) / U;
 }
 
-template <typename T, int D, int G>
+// kAppend: the decode step fused with the cache update -- each request's new
+// key/value (k_new, v_new) is written as cache row len[b], attended to as that
+// row (copied straight from k_new/v_new), and len[b] advances by one.
+template <typename T, int D, int G, bool kAppend>
 __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, G>::kCtasPerSm)
-    decode_attn_kernel(const T *__restrict__ q, const T *__restrict__ kc,
-                       const T *__restrict__ vc, const int64_t *__restrict__ cache_off,
-                       const int32_t *__restrict__ len_in, T *__restrict__ out, float qscale,
-                       int B, int H_kv, float *__restrict__ partials, int slot_floats,
-                       int *__restrict__ counters, int *__restrict__ err) {
+    decode_attn_kernel(const T *__restrict__ q, const T *__restrict__ k_new,
+                       const T *__restrict__ v_new, T *__restrict__ kc, T *__restrict__ vc,
+                       const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
+                       T *__restrict__ out, float qscale, int B, int H_kv,
+                       float *__restrict__ partials, int slot_floats, int *__restrict__ counters,
+                       int *__restrict__ done, int *__restrict__ err) {
     using C = DecodeCfg<T, D, G>;
     constexpr int W = C::kWarps, S = C::kStages, TR = C::kTileRows, RW = C::kRowsPerWarp;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -136,7 +143,9 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     float2 *pbuf = reinterpret_cast<float2 *>(smem + C::kStagesBytes + C::kBarBytes);
     float *mrg = reinterpret_cast<float *>(pbuf + W * RW * G);  // [2][kMergeFloats]
     volatile int *flags = reinterpret_cast<volatile int *>(mrg + 2 * C::kMergeFloats);
-    int64_t *cum = reinterpret_cast<int64_t *>(const_cast<int *>(flags) + 4);
+    int64_t *cum = reinterpret_cast<int64_t *>(const_cast<int *>(flags) + 4);  // [B+1]
+    int64_t *offs = cum + (B + 1);                                             // [B+1]
+    int32_t *newrow = reinterpret_cast<int32_t *>(offs + (B + 1));             // [B]
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
@@ -144,16 +153,28 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
 
     // ---- 1. per-request lengths (clamped to capacity) and their prefix sums
     for (int b = tid; b < B; b += blockDim.x) {
-        const int64_t cap = cache_off[b + 1] - cache_off[b];
-        int64_t L = len_in[b];
-        if (cap < 0 || cache_off[b] < 0) {
+        const int64_t o0 = cache_off[b], o1 = cache_off[b + 1];
+        const int64_t cap = o1 - o0;
+        int64_t L = len[b];
+        int32_t nr = -1;
+        if (cap < 0 || o0 < 0) {
             if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
             L = 0;
         } else if (L < 0 || L > cap) {
             if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_CAPACITY);
             L = L < 0 ? 0 : cap;
+        } else if (kAppend) {
+            if (L < cap) {
+                nr = (int32_t)L;  // the new token becomes row L ...
+                L += 1;           // ... and is attended to
+            } else if (blockIdx.x == 0) {
+                report_error(err, SPEECHKV_ERR_CAPACITY);  // full: attend without it
+            }
         }
         cum[b + 1] = L;
+        offs[b] = o0;
+        if (b == B - 1) offs[B] = o1;
+        newrow[b] = nr;
     }
     if (tid == 0) {
         cum[0] = 0;
@@ -185,6 +206,35 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     }
     __syncthreads();
 
+    if (kAppend) {
+        // every CTA has read len[] once it passes the barrier above; the last
+        // one to get here advances len[] of the requests that took a token
+        if (tid == 0) {
+            if (atomic_add_acq_rel_gpu(done, 1) == (int)gridDim.x - 1) {
+                for (int b = 0; b < B; b++)
+                    if (newrow[b] >= 0) len[b] = newrow[b] + 1;
+                *done = 0;
+            }
+        }
+        // write the new tokens into their cache rows (nothing in this kernel
+        // reads those rows from the cache: the new row is taken from k_new/v_new)
+        constexpr int kVec = 16 / (int)sizeof(T);
+        const int nvec = H_kv * D / kVec;  // 16-byte vectors per token
+        for (int b = blockIdx.x; b < B; b += gridDim.x) {
+            const int32_t nr = newrow[b];
+            if (nr < 0) continue;
+            const int64_t cap = offs[b + 1] - offs[b];
+            for (int i = tid; i < 2 * nvec; i += blockDim.x) {
+                const int tensor = i >= nvec;
+                const int e = (i - tensor * nvec) * kVec;
+                const int hh = e / D, col = e - hh * D;
+                const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
+                T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D + col;
+                copy_bytes<16>(dst, src);
+            }
+        }
+    }
+
     // ---- 2. empty requests get a zero output (softmax over nothing)
     for (int b = blockIdx.x; b < B; b += gridDim.x) {
         if (cum[b + 1] != cum[b]) continue;
@@ -208,8 +258,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         bool stop = false;
         for (int64_t u = u0; u < u1 && !stop;) {
             const Piece p = piece_at(cum, B, H_kv, u, u1);
-            const int64_t cap = cache_off[p.b + 1] - cache_off[p.b];
-            const int64_t base = cache_off[p.b] * H_kv + (int64_t)p.h * cap;
+            const int64_t cap = offs[p.b + 1] - offs[p.b];
+            const int64_t base = offs[p.b] * H_kv + (int64_t)p.h * cap;
+            // with kAppend, row nr of this (request, head) comes from k_new/v_new
+            const int64_t nr = kAppend ? (int64_t)newrow[p.b] : -1;
             for (int64_t t = p.t0; t < p.t1; t += TR) {
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
@@ -224,8 +276,22 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 const bool first = (t == p.t0);
                 unsigned char *dst = stages + (size_t)stage * C::kStageBytes;
                 mbar_arrive_expect_tx(&full_bar[stage], 2 * bytes + (first ? C::kQBytes : 0));
-                bulk_g2s(dst, kc + (base + t) * D, bytes, &full_bar[stage]);
-                bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, bytes, &full_bar[stage]);
+                if (kAppend && nr >= t && nr < t + rows) {
+                    // the tile ends with the new token: cached rows, then one
+                    // row from k_new / v_new (always the last row of the run)
+                    const uint32_t cached = (uint32_t)(nr - t) * C::kRowBytes;
+                    if (cached) {
+                        bulk_g2s(dst, kc + (base + t) * D, cached, &full_bar[stage]);
+                        bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, cached, &full_bar[stage]);
+                    }
+                    const int64_t src = ((int64_t)p.b * H_kv + p.h) * D;
+                    bulk_g2s(dst + cached, k_new + src, C::kRowBytes, &full_bar[stage]);
+                    bulk_g2s(dst + C::kTileBytes + cached, v_new + src, C::kRowBytes,
+                             &full_bar[stage]);
+                } else {
+                    bulk_g2s(dst, kc + (base + t) * D, bytes, &full_bar[stage]);
+                    bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, bytes, &full_bar[stage]);
+                }
                 if (first)
                     bulk_g2s(dst + 2 * C::kTileBytes, q + ((int64_t)p.b * H_q + p.h * G) * D,
                              C::kQBytes, &full_bar[stage]);
@@ -549,11 +615,11 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     }
 }
 
-template <typename T, int D, int G>
+template <typename T, int D, int G, bool kAppend>
 cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) {
     using C = DecodeCfg<T, D, G>;
-    auto kern = decode_attn_kernel<T, D, G>;
-    static int configured_device_mask = 0;  // devices with the smem attribute set
+    auto kern = decode_attn_kernel<T, D, G, kAppend>;
+    static int configured_device_mask = 0;  // devices with the smem attributes set
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -563,26 +629,26 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)C::smem_bytes(SPEECHKV_MAX_BATCH));
         if (e != cudaSuccess) return e;
-        // all of the unified L1/shared storage as shared memory, so that
-        // kCtasPerSm CTAs fit on an SM
+        // all of the unified L1/shared storage as shared memory
         e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
         if (e != cudaSuccess) return e;
         if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
     }
     const float qscale = a.scale * 1.4426950408889634f;  // log2(e): scores in base 2
     kern<<<grid, C::kThreads, C::smem_bytes(a.B), stream>>>(
-        static_cast<const T *>(a.q), static_cast<const T *>(a.k_cache),
-        static_cast<const T *>(a.v_cache), a.cache_off, a.len, static_cast<T *>(a.out), qscale,
-        a.B, a.H_kv, a.partials, decode_slot_floats(D, G), a.counters, a.err);
+        static_cast<const T *>(a.q), static_cast<const T *>(a.k_new),
+        static_cast<const T *>(a.v_new), static_cast<T *>(a.k_cache),
+        static_cast<T *>(a.v_cache), a.cache_off, a.len, static_cast<T *>(a.out), qscale, a.B,
+        a.H_kv, a.partials, decode_slot_floats(D, G), a.counters, a.done, a.err);
     return cudaGetLastError();
 }
 
-// Resident CTAs per SM for a batch of B requests (the length table in shared
-// memory grows with B).
+// Resident CTAs per SM for a batch of B requests (the per-request tables in
+// shared memory grow with B).
 template <typename T, int D, int G>
 int occupancy_instance(int B) {
     using C = DecodeCfg<T, D, G>;
-    auto kern = decode_attn_kernel<T, D, G>;
+    auto kern = decode_attn_kernel<T, D, G, false>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)C::smem_bytes(SPEECHKV_MAX_BATCH)) != cudaSuccess ||
         cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100) !=
@@ -603,8 +669,8 @@ bool decode_supported(speechkv_dtype dtype, int d, int group) {
 }
 
 int decode_slot_floats(int d, int group) {
-    const int f = 2 * group + group * d;
-    return (f + 3) & ~3;  // keep slots 16-byte aligned
+    const int f = group * d + 2 * group;  // o [G][d], then m [G] and l [G]
+    return (f + 3) & ~3;                  // keep slots 16-byte aligned
 }
 
 #define SPEECHKV_DECODE_CASES(X)                                            \
@@ -628,9 +694,11 @@ int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B) {
 
 cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream) {
     const int group = a.H_q / a.H_kv;
-#define X(T, D, G)                                                  \
-    if (a.dtype == dtype_of<T>() && a.d == D && group == G)         \
-        return launch_instance<T, D, G>(a, grid, stream);
+    const bool append = a.k_new != nullptr;
+#define X(T, D, G)                                                               \
+    if (a.dtype == dtype_of<T>() && a.d == D && group == G)                      \
+        return append ? launch_instance<T, D, G, true>(a, grid, stream)          \
+                      : launch_instance<T, D, G, false>(a, grid, stream);
     SPEECHKV_DECODE_CASES(X)
 #undef X
     return cudaErrorInvalidValue;

@@ -37,15 +37,18 @@ struct AppendArgs {
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream);
 
 struct DecodeArgs {
-    const void *q, *k_cache, *v_cache;
+    const void *q;
+    const void *k_new, *v_new;  // non-null: fused append (speechkv_decode_step)
+    void *k_cache, *v_cache;
     const int64_t *cache_off;
-    const int32_t *len;
+    int32_t *len;  // read; with a fused append also advanced
     void *out;
     float scale;  // > 0
     int32_t B, H_q, H_kv, d;
     speechkv_dtype dtype;
     float *partials;   // [grid + B*H_kv][slot_floats]
     int *counters;     // [B*H_kv]
+    int *done;         // CTAs past the prologue (fused append only)
     int *err;
 };
 

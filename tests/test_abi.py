@@ -20,7 +20,7 @@ def _declared():
 
 def test_header_declares_the_path():
     names = _declared()
-    for n in ("speechkv_pool", "speechkv_append", "speechkv_decode_attn",
+    for n in ("speechkv_pool", "speechkv_append", "speechkv_decode_attn", "speechkv_decode_step",
               "speechkv_compressed_len", "speechkv_decode_workspace_size",
               "speechkv_check_device_error", "speechkv_status_string"):
         assert n in names
@@ -82,7 +82,8 @@ def test_workspace_size_explicit_grid():
     lib = sk.load()
     B, H_q, H_kv, d, grid = 8, 16, 8, 128, 152
     n = lib.speechkv_decode_workspace_size(B, H_q, H_kv, d, grid)
-    slot = 2 * 2 + 2 * 128
-    assert n == 256 + (grid + B * H_kv) * slot * 4
+    slot = 2 * 128 + 2 * 2                        # o [G][d], m [G], l [G]
+    counters = -(-(B * H_kv + 1) * 4 // 256) * 256  # per (request, head) + 1
+    assert n == counters + (grid + B * H_kv) * slot * 4
     assert lib.speechkv_decode_workspace_size(B, 7, H_kv, d, grid) == 0
     assert lib.speechkv_decode_workspace_size(B, H_q, H_kv, 100, grid) == 0

@@ -285,18 +285,23 @@ def test_invalid_arguments_return_status(sk):
 # --------------------------------------------------------------------------
 # whole path: prefill pooling, then append + attend for several steps
 # --------------------------------------------------------------------------
-def _run_steps(sk, oracle, wl, layers, steps):
+def _run_steps(sk, oracle, wl, layers, steps, fused=False, grid=0):
     for layer in layers:
         L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=steps)
         oc = H.oracle_prefill(oracle, wl, layer, steps, ks, vs, gate)
-        ws = _ws(sk, wl)
+        ws = _ws(sk, wl, grid)
         store = oracle.STORE_F32 if wl.dtype == "f32" else oracle.STORE_BF16
         for b in range(wl.B):
             assert int(L.len[b]) == oc[b][2]
         for step in range(steps):
             q, kn, vn = inputs.step_qkv(wl, layer, step)
-            sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
-            out = _decode(sk, wl, L, q.cuda(), layer, ws=ws)
+            if fused:
+                out = torch.empty_like(q, device="cuda")
+                sk.decode_step(q.cuda(), kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, out,
+                               ws, wl.w, layer, wl.l0, grid_ctas=grid)
+            else:
+                sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
+                out = _decode(sk, wl, L, q.cuda(), layer, ws=ws, grid=grid)
             ref = []
             for b in range(wl.B):
                 Kc, Vc, n = oc[b]
@@ -328,13 +333,67 @@ def test_end_to_end_ragged_small(sk, oracle):
 
 
 # --------------------------------------------------------------------------
+# fused step: append + decode attention in one launch
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("grid", [0, 1, 7, 300])
+def test_fused_step_tiny_fp32(sk, oracle, grid):
+    _run_steps(sk, oracle, inputs.tiny_fp32(), layers=[0], steps=8, fused=True, grid=grid)
+
+
+def test_fused_step_qwen_and_ragged(sk, oracle):
+    wl = inputs.qwen_single()
+    _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=4, fused=True)
+    wl = inputs.qwen_ragged(B=6)
+    _run_steps(sk, oracle, wl, layers=[wl.l0], steps=3, fused=True)
+
+
+def test_fused_step_matches_separate_calls_and_writes_cache(sk):
+    """decode_step leaves the same cache and lengths as append + decode_attn
+    (bit-exact) and gives the same output up to summation order."""
+    wl = _wl("bf16", (0, 0, 3), (375, 40, 9), (32, 5, 0), (3, 0, 1), w=4, H_q=16, H_kv=8,
+             d=128)
+    A, _ = H.gpu_prefill(wl, 0, extra_rows=3)
+    Bc, _ = H.gpu_prefill(wl, 0, extra_rows=3)
+    wsA, wsB = _ws(sk, wl), _ws(sk, wl)
+    for step in range(3):
+        q, kn, vn = (x.cuda() for x in inputs.step_qkv(wl, 0, step))
+        sk.append(kn, vn, A.k, A.v, A.cache_off, A.len, wl.w, 0, wl.l0)
+        outA = _decode(sk, wl, A, q, 0, ws=wsA)
+        outB = torch.empty_like(q)
+        sk.decode_step(q, kn, vn, Bc.k, Bc.v, Bc.cache_off, Bc.len, outB, wsB, wl.w, 0, wl.l0)
+        assert torch.equal(A.len, Bc.len)
+        assert torch.equal(A.k, Bc.k) and torch.equal(A.v, Bc.v)
+        H.assert_close(H.f64(outB), H.f64(outA), "bf16", f"step {step}")
+    assert sk.check_device_error() == sk.OK
+
+
+def test_fused_step_full_cache(sk, oracle):
+    """A full cache takes no token: CAPACITY is reported, len stays, and the
+    output is attention over the cached rows alone."""
+    wl = _wl("bf16", (0, 0), (20, 12), (2, 3), w=4, H_q=8, H_kv=4, d=128)
+    L, _ = H.gpu_prefill(wl, 0, extra_rows=0)       # capacity == rows: full
+    q, kn, vn = (x.cuda() for x in inputs.step_qkv(wl, 0, 0))
+    lens, kbefore = L.len.clone(), L.k.clone()
+    out = torch.empty_like(q)
+    sk.decode_step(q, kn, vn, L.k, L.v, L.cache_off, L.len, out, _ws(sk, wl), wl.w, 0, wl.l0)
+    assert sk.check_device_error() == sk.ERR_CAPACITY
+    assert torch.equal(L.len, lens) and torch.equal(L.k, kbefore)
+    H.assert_close(H.f64(out), _oracle_attn_on_gpu_cache(oracle, wl, L, q), "bf16", "full")
+
+
+# --------------------------------------------------------------------------
 # full benchmark sizes, sampled against the oracle
 # --------------------------------------------------------------------------
-def _sampled_full_size(sk, oracle, wl, layer, samples):
+def _sampled_full_size(sk, oracle, wl, layer, samples, fused=False):
     L, _ = H.gpu_prefill(wl, layer, extra_rows=1)
     q, kn, vn = inputs.step_qkv(wl, layer, 0)
-    sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
-    out = _decode(sk, wl, L, q.cuda(), layer)
+    if fused:
+        out = torch.empty_like(q, device="cuda")
+        sk.decode_step(q.cuda(), kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, out,
+                       _ws(sk, wl), wl.w, layer, wl.l0)
+    else:
+        sk.append(kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, wl.w, layer, wl.l0)
+        out = _decode(sk, wl, L, q.cuda(), layer)
     assert sk.check_device_error() == sk.OK
     lens = L.len.cpu().numpy()
     for b in samples:
@@ -351,6 +410,12 @@ def test_full_size_long_audio_sampled(sk, oracle, minutes, w):
     _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 5])
 
 
-def test_full_size_ragged_sampled(sk, oracle):
+@pytest.mark.parametrize("fused", [False, True])
+def test_full_size_ragged_sampled(sk, oracle, fused):
     wl = inputs.qwen_ragged()
-    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 17, 64, 127])
+    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 17, 64, 127], fused=fused)
+
+
+def test_full_size_long_audio_fused(sk, oracle):
+    wl = inputs.qwen_long_audio(20, 4, generated=64)
+    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[3], fused=True)
