@@ -224,6 +224,7 @@ class DecodeModel:
                     sk.append(kn[i], vn[i], self.k[i], self.v[i], self.off[i], self.len[i],
                               wl.w, layer, wl.l0)
         self.rows0 = [self.len[i].cpu().tolist() for i in range(L)]
+        self.next_step = [0] * L
         # per-step inputs, resident before the timed region
         self.q = inputs.device_normal((steps_total, L, B, Hq, d), self.dtype, device, wl.seed, seed_key, 6)
         self.kn = inputs.device_normal((steps_total, L, B, Hk, d), self.dtype, device, wl.seed, seed_key, 7)
@@ -233,25 +234,29 @@ class DecodeModel:
         status = sk.check_device_error()
         assert status == sk.OK, sk.status_string(status)
 
-    def launch_step(self, s: int, events=None, fused: bool = True):
-        """One decode step over all layers: speechkv_decode_step (append fused
-        into the attention launch), or speechkv_append + speechkv_decode_attn."""
+    def launch_layer(self, i: int, fused: bool = True):
+        """One decode step of layer position i: speechkv_decode_step (append
+        fused into the attention launch) or speechkv_append followed by
+        speechkv_decode_attn.  Uses the layer's next step of inputs and
+        returns the algorithmic bytes of its decode-attention launch."""
         wl, sk = self.wl, self.sk
-        for i, layer in enumerate(self.layers):
-            if not fused:
-                sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
-                          self.len[i], wl.w, layer, wl.l0)
-            if events is not None:
-                events[i][0].record()
-            if fused:
-                sk.decode_step(self.q[s, i], self.kn[s, i], self.vn[s, i], self.k[i], self.v[i],
-                               self.off[i], self.len[i], self.out[i], self.ws, wl.w, layer,
-                               wl.l0)
-            else:
-                sk.decode_attn(self.q[s, i], self.k[i], self.v[i], self.off[i], self.len[i],
-                               self.out[i], self.ws, wl.w, layer, wl.l0, wl.H_kv)
-            if events is not None:
-                events[i][1].record()
+        s, layer = self.next_step[i], self.layers[i]
+        if fused:
+            sk.decode_step(self.q[s, i], self.kn[s, i], self.vn[s, i], self.k[i], self.v[i],
+                           self.off[i], self.len[i], self.out[i], self.ws, wl.w, layer, wl.l0)
+        else:
+            sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
+                      self.len[i], wl.w, layer, wl.l0)
+            sk.decode_attn(self.q[s, i], self.k[i], self.v[i], self.off[i], self.len[i],
+                           self.out[i], self.ws, wl.w, layer, wl.l0, wl.H_kv)
+        self.next_step[i] = s + 1
+        return self.attn_bytes([r + s + 1 for r in self.rows0[i]], fused)
+
+    def launch_step(self, positions=None, fused: bool = True) -> int:
+        """One decode step over the given layer positions (default: all, in
+        model order).  Returns the algorithmic bytes of its attention launches."""
+        positions = range(len(self.layers)) if positions is None else positions
+        return sum(self.launch_layer(i, fused) for i in positions)
 
     def attn_bytes(self, rows_per_req, fused: bool = True) -> int:
         """Algorithmic bytes of one decode-attention launch: every K and V row
@@ -267,25 +272,24 @@ class DecodeModel:
             setattr(self, name, None)
 
 
-def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist: Dist,
-              clocks: ClockSampler | None, kernel_events: bool = True, fused: bool = True):
-    """Capture `steps` decode steps in CUDA graphs of `chunk` steps, then replay
-    them as the timed region.  Returns (region_ms, per-layer attn ms lists)."""
+def run_timed(model: DecodeModel, positions, steps: int, chunk: int, dist: Dist,
+              clocks: ClockSampler | None, fused: bool = True):
+    """Capture `steps` decode steps over the layer positions in CUDA graphs of
+    `chunk` steps, then replay them back to back as the timed region (CUDA
+    events on the launching stream around it, max over ranks).  Returns
+    (region_ms, algorithmic bytes of all attention launches, launches)."""
     import torch
-    L = len(model.layers)
-    graphs, evs = [], []
-    s = first_step
-    while s < first_step + steps:
-        n = min(chunk, first_step + steps - s)
-        ev = [[[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)]
-               for _ in range(L)] for _ in range(n)] if kernel_events else None
+    graphs, nbytes, launches = [], 0, 0
+    done = 0
+    while done < steps:
+        n = min(chunk, steps - done)
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            for i in range(n):
-                model.launch_step(s + i, ev[i] if ev else None, fused=fused)
+            for _ in range(n):
+                nbytes += model.launch_step(positions, fused=fused)
+                launches += len(positions) * (1 if fused else 2)
         graphs.append(g)
-        evs.append(ev)
-        s += n
+        done += n
     dist.barrier()
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t0 = time.time()
@@ -299,68 +303,58 @@ def run_timed(model: DecodeModel, first_step: int, steps: int, chunk: int, dist:
     if clocks:
         clocks.mark(t0, t1)
     region_ms = dist.max(start.elapsed_time(end))
-    per_layer = [[] for _ in range(L)]
-    if kernel_events:
-        for ev in evs:
-            for step_ev in ev:
-                for layer in range(L):
-                    per_layer[layer].append(step_ev[layer][0].elapsed_time(step_ev[layer][1]))
     del graphs
-    return region_ms, per_layer
+    return region_ms, nbytes, launches
 
 
 def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int,
             layers=None, fused: bool = True):
-    """Build the model for `wl`, run warm-up steps eagerly, then two timed
-    passes of `steps` graph-replayed decode steps each: the first with no
-    events inside the graphs (the step time), the second with CUDA events
-    around every decode-attention launch (per-kernel durations for the
-    roofline).  Returns a result dict."""
+    """Build the model for `wl`, run warm-up steps eagerly, then three timed
+    passes of `steps` graph-replayed decode steps, none with events inside the
+    graphs: (A) every layer in model order -- the decode step; (B) the pooled
+    layers only; (C) the full-resolution layers only -- per-layer times of
+    the two kinds.  Returns a result dict."""
     import torch
-    model = DecodeModel(wl, steps_total=warmup + 2 * steps, seed_key=seed_key, layers=layers)
-    for s in range(warmup):
-        model.launch_step(s, fused=fused)
+    model = DecodeModel(wl, steps_total=warmup + 3 * steps, seed_key=seed_key, layers=layers)
+    L = len(model.layers)
+    comp = [i for i, layer in enumerate(model.layers) if layer >= wl.l0]
+    full = [i for i, layer in enumerate(model.layers) if layer < wl.l0]
+    for _ in range(warmup):
+        model.launch_step(fused=fused)
     torch.cuda.synchronize()
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
-    L = len(model.layers)
-    region_ms, _ = run_timed(model, warmup, steps, chunk, dist, clocks, kernel_events=False,
-                             fused=fused)
-    base_rows = [[model.rows0[i][b] + warmup + steps for b in range(wl.B)] for i in range(L)]
-    events_region_ms, per_layer = run_timed(model, warmup + steps, steps, chunk, dist, clocks,
-                                            kernel_events=True, fused=fused)
+    ms_a, bytes_a, launches_a = run_timed(model, list(range(L)), steps, chunk, dist, clocks,
+                                          fused)
+    per_kind = {}
+    for kind, pos in (("compressed", comp), ("full", full)):
+        if pos:
+            ms, nb, _ = run_timed(model, pos, steps, chunk, dist, clocks, fused)
+            per_kind[kind] = (ms * 1e3 / (steps * len(pos)), nb / (ms * 1e-3) / 1e9,
+                              nb / (steps * len(pos)))
+        else:
+            per_kind[kind] = (float("nan"),) * 3
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
-    comp = [i for i, layer in enumerate(model.layers) if layer >= wl.l0]
-    full = [i for i, layer in enumerate(model.layers) if layer < wl.l0]
-    mean = lambda xs: sum(xs) / len(xs) if xs else float("nan")  # noqa: E731
-    ratio = lambda a, b: a / b if b else float("nan")  # noqa: E731
-    attn_ms = {i: mean(per_layer[i]) for i in range(L)}
-    # algorithmic bytes: rows after step t's append are base + t + 1
-    bytes_total = {i: sum(model.attn_bytes([r + t + 1 for r in base_rows[i]], fused)
-                          for t in range(steps)) for i in range(L)}
-    time_total = {i: sum(per_layer[i]) for i in range(L)}
     res = {
         "minutes": wl.T[0] * 80 / 60000.0, "w": wl.w, "B": wl.B,
-        "step_us": region_ms * 1e3 / steps,
-        "us_per_step_per_layer": region_ms * 1e3 / steps / L,
-        "attn_us_per_layer": mean([attn_ms[l] for l in range(L)]) * 1e3,
-        "attn_us_compressed_layer": mean([attn_ms[l] for l in comp]) * 1e3,
-        "attn_us_full_layer": mean([attn_ms[l] for l in full]) * 1e3,
-        "attn_gbs_compressed_layer": ratio(sum(bytes_total[i] for i in comp),
-                                           sum(time_total[i] for i in comp) * 1e-3) / 1e9,
-        "attn_gbs_all_layers": ratio(sum(bytes_total.values()),
-                                     sum(time_total.values()) * 1e-3) / 1e9,
-        "attn_bytes_per_launch_compressed": ratio(sum(bytes_total[i] for i in comp),
-                                                  len(comp) * steps),
-        "attn_bytes_per_launch_all": sum(bytes_total.values()) / (L * steps),
-        "pool_us_compressed_layer": mean([model.pool_ms[model.layers[i]] for i in comp]) * 1e3,
-        "pool_us_full_layer": mean([model.pool_ms[model.layers[i]] for i in full]) * 1e3,
-        "gpu_launches": steps * L * (1 if fused else 2),
-        "region_ms": region_ms,
-        "events_pass_step_us": events_region_ms * 1e3 / steps,
-        "path": "speechkv_decode_step (append fused)" if fused else
-                "speechkv_append + speechkv_decode_attn",
+        "path": ("speechkv_decode_step (append fused)" if fused else
+                 "speechkv_append + speechkv_decode_attn"),
+        "step_us": ms_a * 1e3 / steps,
+        "us_per_step_per_layer": ms_a * 1e3 / steps / L,
+        "step_gbs": bytes_a / (ms_a * 1e-3) / 1e9,
+        "attn_bytes_per_launch_all": bytes_a / (steps * L),
+        "attn_us_compressed_layer": per_kind["compressed"][0],
+        "attn_gbs_compressed_layer": per_kind["compressed"][1],
+        "attn_bytes_per_launch_compressed": per_kind["compressed"][2],
+        "attn_us_full_layer": per_kind["full"][0],
+        "attn_gbs_full_layer": per_kind["full"][1],
+        "pool_us_compressed_layer": (sum(model.pool_ms[model.layers[i]] for i in comp) /
+                                     len(comp) * 1e3 if comp else float("nan")),
+        "pool_us_full_layer": (sum(model.pool_ms[model.layers[i]] for i in full) /
+                               len(full) * 1e3 if full else float("nan")),
+        "gpu_launches": launches_a,
+        "region_ms": ms_a,
     }
     model.free()
     del model
@@ -637,11 +631,12 @@ def main():
             w1 = w1_by_min.get(minutes)
             sweep.append({
                 "audio_min": minutes, "w": w,
-                "attn_us_per_layer": round(r["attn_us_per_layer"], 2),
+                "us_per_step_per_layer": round(r["us_per_step_per_layer"], 2),
+                "step_gbs": round(r["step_gbs"], 1),
                 "attn_us_compressed_layer": round(r["attn_us_compressed_layer"], 2),
                 "attn_gbs_compressed_layer": round(r["attn_gbs_compressed_layer"], 1),
-                "us_per_step_per_layer": round(r["us_per_step_per_layer"], 2),
-                "w1_attn_us_full_layer": round(w1["attn_us_compressed_layer"], 2) if w1 else None,
+                "w1_us_per_step_per_layer": round(w1["us_per_step_per_layer"], 2) if w1 else None,
+                "w1_attn_us_same_layer": round(w1["attn_us_compressed_layer"], 2) if w1 else None,
                 "speedup_vs_w1_compressed_layer": (round(w1["attn_us_compressed_layer"] /
                                                          r["attn_us_compressed_layer"], 3)
                                                    if w1 else None),
@@ -655,7 +650,7 @@ def main():
 
     if dist.rank == 0:
         peak, peak_kind = measured_peak()
-        ach = main_res["attn_gbs_all_layers"]
+        ach = main_res["step_gbs"]
         line = {
             "metric": METRIC,
             "value": round(main_res["us_per_step_per_layer"], 3),
@@ -675,9 +670,12 @@ def main():
                 "frac": round(ach / peak, 4), "peak_kind": peak_kind,
                 "traffic": profiled_traffic(main_res["attn_bytes_per_launch_all"]),
                 "kernel": ("decode_attn_kernel (fused append, bf16, d=128, group 2) of "
-                           "speechkv_decode_step, all 28 layers"),
+                           "speechkv_decode_step: the only kernel of the step"),
+                "achieved_from": "algorithmic bytes of all launches of the timed steps / "
+                                 "timed-region time (all 28 layers, launch gaps included)",
                 "algorithmic_bytes_per_launch": round(main_res["attn_bytes_per_launch_all"]),
                 "compressed_layers": {
+                    "us_per_launch": round(main_res["attn_us_compressed_layer"], 3),
                     "achieved": round(main_res["attn_gbs_compressed_layer"], 1),
                     "frac": round(main_res["attn_gbs_compressed_layer"] / peak, 4),
                     "frac_of_8tbs_nominal": round(main_res["attn_gbs_compressed_layer"] / 8000, 4),
@@ -698,9 +696,7 @@ def main():
             "speedup_vs_w1": ({
                 "decode_attn_compressed_layer": round(w1_res["attn_us_compressed_layer"] /
                                                       main_res["attn_us_compressed_layer"], 3),
-                "decode_attn_28_layers": round(w1_res["attn_us_per_layer"] /
-                                               main_res["attn_us_per_layer"], 3),
-                "decode_step": round(w1_res["step_us"] / main_res["step_us"], 3),
+                "decode_step_28_layers": round(w1_res["step_us"] / main_res["step_us"], 3),
             } if w1_res else None),
             "by_audio_len": sweep or None,
         }

@@ -206,35 +206,6 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     }
     __syncthreads();
 
-    if (kAppend) {
-        // every CTA has read len[] once it passes the barrier above; the last
-        // one to get here advances len[] of the requests that took a token
-        if (tid == 0) {
-            if (atomic_add_acq_rel_gpu(done, 1) == (int)gridDim.x - 1) {
-                for (int b = 0; b < B; b++)
-                    if (newrow[b] >= 0) len[b] = newrow[b] + 1;
-                *done = 0;
-            }
-        }
-        // write the new tokens into their cache rows (nothing in this kernel
-        // reads those rows from the cache: the new row is taken from k_new/v_new)
-        constexpr int kVec = 16 / (int)sizeof(T);
-        const int nvec = H_kv * D / kVec;  // 16-byte vectors per token
-        for (int b = blockIdx.x; b < B; b += gridDim.x) {
-            const int32_t nr = newrow[b];
-            if (nr < 0) continue;
-            const int64_t cap = offs[b + 1] - offs[b];
-            for (int i = tid; i < 2 * nvec; i += blockDim.x) {
-                const int tensor = i >= nvec;
-                const int e = (i - tensor * nvec) * kVec;
-                const int hh = e / D, col = e - hh * D;
-                const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
-                T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D + col;
-                copy_bytes<16>(dst, src);
-            }
-        }
-    }
-
     // ---- 2. empty requests get a zero output (softmax over nothing)
     for (int b = blockIdx.x; b < B; b += gridDim.x) {
         if (cum[b + 1] != cum[b]) continue;
@@ -246,6 +217,39 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int64_t U = (int64_t)H_kv * cum[B];
     const int64_t Cn = U < (int64_t)gridDim.x ? U : (int64_t)gridDim.x;
     const int64_t c = blockIdx.x;
+    if (kAppend && warp == W + 1) {
+        // every CTA has read len[] once past the prologue's barrier; the last
+        // one to get here advances len[] of the requests that took a token
+        int last = 0;
+        if (lane == 0) last = atomic_add_acq_rel_gpu(done, 1) == (int)gridDim.x - 1;
+        last = __shfl_sync(0xffffffffu, last, 0);
+        __syncwarp();
+        if (last) {
+            for (int b = lane; b < B; b += 32)
+                if (newrow[b] >= 0) len[b] = newrow[b] + 1;
+            __syncwarp();
+            if (lane == 0) *done = 0;
+        }
+    }
+    if (kAppend && warp < W) {
+        // write the new tokens into their cache rows (nothing in this kernel
+        // reads those rows from the cache: the new row comes from k_new/v_new)
+        constexpr int kVec = 16 / (int)sizeof(T);
+        const int nvec = H_kv * D / kVec;  // 16-byte vectors per token
+        for (int b = blockIdx.x; b < B; b += gridDim.x) {
+            const int32_t nr = newrow[b];
+            if (nr < 0) continue;
+            const int64_t cap = offs[b + 1] - offs[b];
+            for (int i = tid; i < 2 * nvec; i += W * 32) {
+                const int tensor = i >= nvec;
+                const int e = (i - tensor * nvec) * kVec;
+                const int hh = e / D, col = e - hh * D;
+                const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
+                T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D + col;
+                copy_bytes<16>(dst, src);
+            }
+        }
+    }
     if (c >= Cn) return;
     const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
 
