@@ -234,7 +234,7 @@ class DecodeModel:
         status = sk.check_device_error()
         assert status == sk.OK, sk.status_string(status)
 
-    def launch_layer(self, i: int, fused: bool = True):
+    def launch_layer(self, i: int, fused: bool = True, overlap: bool = False):
         """One decode step of layer position i: speechkv_decode_step (append
         fused into the attention launch) or speechkv_append followed by
         speechkv_decode_attn.  Uses the layer's next step of inputs and
@@ -242,8 +242,11 @@ class DecodeModel:
         wl, sk = self.wl, self.sk
         s, layer = self.next_step[i], self.layers[i]
         if fused:
+            # overlap: the previous kernel on the stream is another layer's
+            # decode step, which writes none of this layer's cache or lengths
             sk.decode_step(self.q[s, i], self.kn[s, i], self.vn[s, i], self.k[i], self.v[i],
-                           self.off[i], self.len[i], self.out[i], self.ws, wl.w, layer, wl.l0)
+                           self.off[i], self.len[i], self.out[i], self.ws, wl.w, layer, wl.l0,
+                           flags=sk.OVERLAP_PRIOR if overlap else 0)
         else:
             sk.append(self.kn[s, i], self.vn[s, i], self.k[i], self.v[i], self.off[i],
                       self.len[i], wl.w, layer, wl.l0)
@@ -254,9 +257,12 @@ class DecodeModel:
 
     def launch_step(self, positions=None, fused: bool = True) -> int:
         """One decode step over the given layer positions (default: all, in
-        model order).  Returns the algorithmic bytes of its attention launches."""
-        positions = range(len(self.layers)) if positions is None else positions
-        return sum(self.launch_layer(i, fused) for i in positions)
+        model order).  Returns the algorithmic bytes of its attention launches.
+        Consecutive fused launches of different layers may overlap
+        (SPEECHKV_OVERLAP_PRIOR); a single layer never overlaps itself."""
+        positions = list(range(len(self.layers))) if positions is None else list(positions)
+        overlap = fused and len(positions) > 1
+        return sum(self.launch_layer(i, fused, overlap) for i in positions)
 
     def attn_bytes(self, rows_per_req, fused: bool = True) -> int:
         """Algorithmic bytes of one decode-attention launch: every K and V row

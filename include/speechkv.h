@@ -68,6 +68,20 @@ typedef enum { SPEECHKV_F32 = 0, SPEECHKV_BF16 = 1 } speechkv_dtype;
 /* Largest batch speechkv_decode_attn / _step accept (their per-CTA tables). */
 #define SPEECHKV_MAX_BATCH 512
 
+/*
+ * Flag of speechkv_decode_attn / speechkv_decode_step.  The decode kernels
+ * are launched with programmatic dependent launch, so they may begin while
+ * the previous kernel on the stream retires.  By default they wait for that
+ * kernel before reading anything.  SPEECHKV_OVERLAP_PRIOR declares that the
+ * previous kernel on `stream` writes none of this call's caches, len or
+ * cache_off (it may produce q, k_new and v_new, and may use the same
+ * workspace): the call then reads the lengths and starts streaming the
+ * cached rows at once, and waits for the previous kernel only before
+ * reading q / k_new / v_new and before any write.  A kernel that precedes
+ * it without the launch attribute is simply waited for, as usual.
+ */
+#define SPEECHKV_OVERLAP_PRIOR 1u
+
 /* Human-readable name of a status (static string, never NULL). */
 const char *speechkv_status_string(speechkv_status status);
 
@@ -182,6 +196,7 @@ size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv,
  *              first use; every call leaves its counters at zero again.
  *              Calls that run concurrently need separate workspaces.  After
  *              a device error, zero it again.
+ * flags        0 or SPEECHKV_OVERLAP_PRIOR (see above).
  */
 speechkv_status speechkv_decode_attn(const void *q, const void *k_cache,
                                      const void *v_cache,
@@ -192,7 +207,7 @@ speechkv_status speechkv_decode_attn(const void *q, const void *k_cache,
                                      int32_t layer, int32_t l0,
                                      int32_t grid_ctas, void *workspace,
                                      size_t workspace_bytes,
-                                     speechkv_dtype dtype,
+                                     speechkv_dtype dtype, uint32_t flags,
                                      cudaStream_t stream);
 
 /*
@@ -221,7 +236,8 @@ speechkv_status speechkv_decode_step(const void *q, const void *k_new,
                                      int32_t d, int32_t w, int32_t layer,
                                      int32_t l0, int32_t grid_ctas,
                                      void *workspace, size_t workspace_bytes,
-                                     speechkv_dtype dtype, cudaStream_t stream);
+                                     speechkv_dtype dtype, uint32_t flags,
+                                     cudaStream_t stream);
 
 /*
  * Synchronises `stream`, then reads and clears the current device's error

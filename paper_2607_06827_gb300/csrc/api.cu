@@ -116,9 +116,11 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
                               int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
                               int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
                               int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                              speechkv_dtype dtype, cudaStream_t stream, bool append) {
+                              speechkv_dtype dtype, uint32_t flags, cudaStream_t stream,
+                              bool append) {
     if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
-        grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale))
+        grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale) ||
+        (flags & ~SPEECHKV_OVERLAP_PRIOR))
         return SPEECHKV_ERR_INVALID_ARG;
     if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
     if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
@@ -161,6 +163,7 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
     a.partials = reinterpret_cast<float *>(static_cast<char *>(workspace) +
                                            counters_bytes(B, H_kv));
     a.err = s->err;
+    a.overlap = (flags & SPEECHKV_OVERLAP_PRIOR) != 0;
     return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
                                                                    : SPEECHKV_ERR_CUDA;
 }
@@ -283,12 +286,12 @@ speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const v
                                      float scale, int32_t B, int32_t H_q, int32_t H_kv,
                                      int32_t d, int32_t w, int32_t layer, int32_t l0,
                                      int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                                     speechkv_dtype dtype, cudaStream_t stream) {
+                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
     // the caches and len are only read on this path
     return decode_common(q, nullptr, nullptr, const_cast<void *>(k_cache),
                          const_cast<void *>(v_cache), cache_off, const_cast<int32_t *>(len), out,
                          scale, B, H_q, H_kv, d, w, layer, l0, grid_ctas, workspace,
-                         workspace_bytes_in, dtype, stream, false);
+                         workspace_bytes_in, dtype, flags, stream, false);
 }
 
 speechkv_status speechkv_decode_step(const void *q, const void *k_new, const void *v_new,
@@ -296,10 +299,10 @@ speechkv_status speechkv_decode_step(const void *q, const void *k_new, const voi
                                      int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
                                      int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
                                      int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                                     speechkv_dtype dtype, cudaStream_t stream) {
+                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
     return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
                          H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
-                         stream, true);
+                         flags, stream, true);
 }
 
 speechkv_status speechkv_check_device_error(cudaStream_t stream) {

@@ -197,6 +197,20 @@ __device__ __forceinline__ void fence_proxy_async_shared() {
 }
 
 // ---------------------------------------------------------------------------
+// programmatic dependent launch (kernels launched with the PDL attribute)
+// ---------------------------------------------------------------------------
+// Let the next kernel on the stream (if it was launched with the attribute)
+// be scheduled as this grid's CTAs retire.
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+// Block until the grids this one depends on have completed and their memory
+// operations are visible (a no-op when launched without the attribute).
+__device__ __forceinline__ void griddep_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// ---------------------------------------------------------------------------
 // mbarrier + bulk asynchronous copy (TMA, non-tensor form)
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {

@@ -131,7 +131,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                        const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
                        T *__restrict__ out, float qscale, int B, int H_kv,
                        float *__restrict__ partials, int slot_floats, int *__restrict__ counters,
-                       int *__restrict__ done, int *__restrict__ err) {
+                       int *__restrict__ done, int *__restrict__ err, int overlap) {
     using C = DecodeCfg<T, D, G>;
     constexpr int W = C::kWarps, S = C::kStages, TR = C::kTileRows, RW = C::kRowsPerWarp;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -150,6 +150,16 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
     const int H_q = H_kv * G;
+
+    // Programmatic dependent launch: the next kernel may start as our CTAs
+    // retire.  Unless the caller declared that the previous kernel on the
+    // stream produces at most q, k_new and v_new (overlap != 0), wait for it
+    // before touching anything.  With overlap, the prologue and the bulk
+    // copies of cached rows run first; every read of q / k_new / v_new and
+    // every global write (outputs, cache rows, len, workspace) comes after
+    // griddep_wait(), and every thread waits before it exits.
+    griddep_launch_dependents();
+    if (!overlap) griddep_wait();
 
     // ---- 1. per-request lengths (clamped to capacity) and their prefix sums
     for (int b = tid; b < B; b += blockDim.x) {
@@ -206,17 +216,19 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     }
     __syncthreads();
 
-    // ---- 2. empty requests get a zero output (softmax over nothing)
-    for (int b = blockIdx.x; b < B; b += gridDim.x) {
-        if (cum[b + 1] != cum[b]) continue;
-        for (int i = tid; i < H_q * D; i += blockDim.x)
-            out[(int64_t)b * H_q * D + i] = from_float<T>(0.f);
-    }
-
-    // ---- 3. this CTA's share of the flat (request, head, row) range
+    // ---- 2. this CTA's share of the flat (request, head, row) range
     const int64_t U = (int64_t)H_kv * cum[B];
     const int64_t Cn = U < (int64_t)gridDim.x ? U : (int64_t)gridDim.x;
     const int64_t c = blockIdx.x;
+    if (warp == W + 1) {
+        griddep_wait();
+        // empty requests get a zero output (softmax over nothing)
+        for (int b = blockIdx.x; b < B; b += gridDim.x) {
+            if (cum[b + 1] != cum[b]) continue;
+            for (int i = lane; i < H_q * D; i += 32)
+                out[(int64_t)b * H_q * D + i] = from_float<T>(0.f);
+        }
+    }
     if (kAppend && warp == W + 1) {
         // every CTA has read len[] once past the prologue's barrier; the last
         // one to get here advances len[] of the requests that took a token
@@ -232,6 +244,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         }
     }
     if (kAppend && warp < W) {
+        griddep_wait();
         // write the new tokens into their cache rows (nothing in this kernel
         // reads those rows from the cache: the new row comes from k_new/v_new)
         constexpr int kVec = 16 / (int)sizeof(T);
@@ -250,16 +263,48 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             }
         }
     }
-    if (c >= Cn) return;
+    if (c >= Cn) {
+        griddep_wait();
+        return;
+    }
     const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
 
     if (warp == W) {
         // ================= producer: one lane issues bulk copies ============
-        if (lane != 0) return;
+        if (lane != 0) {
+            griddep_wait();
+            return;
+        }
         int stage = 0;
         uint32_t phase = 0;
         int64_t issued = 0;
         bool stop = false;
+        // Copies of data the previous kernel may produce (queries, new
+        // tokens) wait for it; until then they are queued here.  Only the
+        // first S tiles can be issued before the first stage must be reused,
+        // so the queue holds at most 3 copies per stage.
+        struct Deferred {
+            void *dst;
+            const void *src;
+            uint32_t bytes;
+            uint64_t *bar;
+        };
+        Deferred deferred[3 * S];
+        int ndeferred = 0;
+        bool waited = !overlap;
+        auto copy_prior = [&](void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+            if (waited)
+                bulk_g2s(dst, src, bytes, bar);
+            else
+                deferred[ndeferred++] = Deferred{dst, src, bytes, bar};
+        };
+        auto flush_deferred = [&]() {
+            griddep_wait();
+            waited = true;
+            for (int i = 0; i < ndeferred; i++)
+                bulk_g2s(deferred[i].dst, deferred[i].src, deferred[i].bytes, deferred[i].bar);
+            ndeferred = 0;
+        };
         for (int64_t u = u0; u < u1 && !stop;) {
             const Piece p = piece_at(cum, B, H_kv, u, u1);
             const int64_t cap = offs[p.b + 1] - offs[p.b];
@@ -267,6 +312,8 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             // with kAppend, row nr of this (request, head) comes from k_new/v_new
             const int64_t nr = kAppend ? (int64_t)newrow[p.b] : -1;
             for (int64_t t = p.t0; t < p.t1; t += TR) {
+                // a stage is about to be reused: its queries may be queued
+                if (!waited && issued == S) flush_deferred();
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
                 if (flags[0] || !mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, err) ||
@@ -289,16 +336,16 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                         bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, cached, &full_bar[stage]);
                     }
                     const int64_t src = ((int64_t)p.b * H_kv + p.h) * D;
-                    bulk_g2s(dst + cached, k_new + src, C::kRowBytes, &full_bar[stage]);
-                    bulk_g2s(dst + C::kTileBytes + cached, v_new + src, C::kRowBytes,
-                             &full_bar[stage]);
+                    copy_prior(dst + cached, k_new + src, C::kRowBytes, &full_bar[stage]);
+                    copy_prior(dst + C::kTileBytes + cached, v_new + src, C::kRowBytes,
+                               &full_bar[stage]);
                 } else {
                     bulk_g2s(dst, kc + (base + t) * D, bytes, &full_bar[stage]);
                     bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, bytes, &full_bar[stage]);
                 }
                 if (first)
-                    bulk_g2s(dst + 2 * C::kTileBytes, q + ((int64_t)p.b * H_q + p.h * G) * D,
-                             C::kQBytes, &full_bar[stage]);
+                    copy_prior(dst + 2 * C::kTileBytes, q + ((int64_t)p.b * H_q + p.h * G) * D,
+                               C::kQBytes, &full_bar[stage]);
                 ++issued;
                 if (++stage == S) {
                     stage = 0;
@@ -307,6 +354,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             }
             u += p.t1 - p.t0;
         }
+        if (!waited) flush_deferred();
         // Let the copies still in flight land before the CTA may exit.
         const int64_t first = issued > S ? issued - S : 0;
         for (int64_t k = first; k < issued; k++)
@@ -617,6 +665,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         if (lane == 0) mbar_arrive(&piece_bar[x]);
         u += p.t1 - p.t0;
     }
+    griddep_wait();
 }
 
 template <typename T, int D, int G, bool kAppend>
@@ -639,12 +688,24 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
         if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
     }
     const float qscale = a.scale * 1.4426950408889634f;  // log2(e): scores in base 2
-    kern<<<grid, C::kThreads, C::smem_bytes(a.B), stream>>>(
-        static_cast<const T *>(a.q), static_cast<const T *>(a.k_new),
-        static_cast<const T *>(a.v_new), static_cast<T *>(a.k_cache),
-        static_cast<T *>(a.v_cache), a.cache_off, a.len, static_cast<T *>(a.out), qscale, a.B,
-        a.H_kv, a.partials, decode_slot_floats(D, G), a.counters, a.done, a.err);
-    return cudaGetLastError();
+    // programmatic dependent launch: may begin while the previous kernel on
+    // the stream retires (the kernel orders itself with griddepcontrol)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(C::kThreads);
+    cfg.dynamicSmemBytes = C::smem_bytes(a.B);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<const T *>(a.q),
+                              static_cast<const T *>(a.k_new), static_cast<const T *>(a.v_new),
+                              static_cast<T *>(a.k_cache), static_cast<T *>(a.v_cache),
+                              a.cache_off, a.len, static_cast<T *>(a.out), qscale, a.B, a.H_kv,
+                              a.partials, decode_slot_floats(D, G), a.counters, a.done, a.err,
+                              a.overlap ? 1 : 0);
 }
 
 // Resident CTAs per SM for a batch of B requests (the per-request tables in

@@ -50,6 +50,7 @@ struct DecodeArgs {
     int *counters;     // [B*H_kv]
     int *done;         // CTAs past the prologue (fused append only)
     int *err;
+    bool overlap;      // SPEECHKV_OVERLAP_PRIOR: start before the previous kernel ends
 };
 
 // Whether (dtype, d, group) has a compiled decode kernel.

@@ -18,6 +18,7 @@ LIB_PATH = os.path.join(_PKG, "libspeechkv.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_CAPACITY, ERR_TIMEOUT, ERR_WORKSPACE = range(7)
 F32, BF16 = 0, 1
+OVERLAP_PRIOR = 1  # SPEECHKV_OVERLAP_PRIOR
 MAX_BATCH = 512
 
 # Every function the header declares: name -> (restype, argtypes)
@@ -36,11 +37,11 @@ SIGNATURES = {
     "speechkv_decode_attn": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _F,
                                             _I32, _I32, _I32, _I32, _I32, _I32,
                                             _I32, _I32, _P, _SZ, ctypes.c_int,
-                                            _P]),
+                                            ctypes.c_uint32, _P]),
     "speechkv_decode_step": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _F,
                                             _I32, _I32, _I32, _I32, _I32, _I32,
                                             _I32, _I32, _P, _SZ, ctypes.c_int,
-                                            _P]),
+                                            ctypes.c_uint32, _P]),
     "speechkv_check_device_error": (ctypes.c_int, [_P]),
 }
 
@@ -147,19 +148,21 @@ def new_workspace(B: int, H_q: int, H_kv: int, d: int, grid_ctas: int = 0,
 
 
 def decode_attn(q, k_cache, v_cache, cache_off, length, out, workspace, w: int, layer: int,
-                l0: int, H_kv: int, scale: float = 0.0, grid_ctas: int = 0, stream=None):
+                l0: int, H_kv: int, scale: float = 0.0, grid_ctas: int = 0, flags: int = 0,
+                stream=None):
     """speechkv_decode_attn: q/out [B, H_q, d]; caches in the head-major
     per-request layout; length int32 [B]."""
     B, H_q, d = q.shape
     _check(load().speechkv_decode_attn(
         _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off), _ptr(length), _ptr(out),
         float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas, _ptr(workspace),
-        workspace.numel() * workspace.element_size(), _dtype_code(q), _stream(stream)),
+        workspace.numel() * workspace.element_size(), _dtype_code(q), flags, _stream(stream)),
         "speechkv_decode_attn")
 
 
 def decode_step(q, k_new, v_new, k_cache, v_cache, cache_off, length, out, workspace, w: int,
-                layer: int, l0: int, scale: float = 0.0, grid_ctas: int = 0, stream=None):
+                layer: int, l0: int, scale: float = 0.0, grid_ctas: int = 0, flags: int = 0,
+                stream=None):
     """speechkv_decode_step: append k_new/v_new ([B, H_kv, d]) to the caches
     and attend (q/out [B, H_q, d]) in one launch; length int32 [B] advances."""
     B, H_q, d = q.shape
@@ -167,7 +170,7 @@ def decode_step(q, k_new, v_new, k_cache, v_cache, cache_off, length, out, works
     _check(load().speechkv_decode_step(
         _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off),
         _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas,
-        _ptr(workspace), workspace.numel() * workspace.element_size(), _dtype_code(q),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _dtype_code(q), flags,
         _stream(stream)),
         "speechkv_decode_step")
 

@@ -63,12 +63,16 @@ def test_host_argument_checks_without_gpu():
     z = None
     # decode: bad window, bad head split, unsupported head dim, B = 0 no-op
     args = lambda B, H_q, H_kv, d, w: (z, z, z, z, z, z, 0.0, B, H_q, H_kv, d, w, 0, 0, 0, z, 0,  # noqa: E731
-                                       sk.BF16, z)
+                                       sk.BF16, 0, z)
     assert lib.speechkv_decode_attn(*args(1, 8, 4, 128, 0)) == sk.ERR_INVALID_ARG
     assert lib.speechkv_decode_attn(*args(1, 7, 4, 128, 4)) == sk.ERR_INVALID_ARG
     assert lib.speechkv_decode_attn(*args(1, 8, 4, 96, 4)) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_decode_attn(*args(0, 8, 4, 128, 4)) == sk.OK
     assert lib.speechkv_decode_attn(*args(1, 8, 4, 128, 4)) == sk.ERR_INVALID_ARG  # NULLs
+    step = lambda B, fl: (z,) * 8 + (0.0, B, 8, 4, 128, 4, 0, 0, 0, z, 0, sk.BF16, fl, z)  # noqa: E731
+    assert lib.speechkv_decode_step(*step(0, 0)) == sk.OK
+    assert lib.speechkv_decode_step(*step(1, 0)) == sk.ERR_INVALID_ARG          # NULLs
+    assert lib.speechkv_decode_step(*step(1, 4)) == sk.ERR_INVALID_ARG          # bad flag
     # append / pool
     assert lib.speechkv_append(z, z, z, z, z, z, 1, 8, 128, 4, -1, 0, sk.BF16, z) == sk.ERR_INVALID_ARG
     assert lib.speechkv_append(z, z, z, z, z, z, 0, 8, 128, 4, 0, 0, sk.BF16, z) == sk.OK

@@ -264,9 +264,9 @@ def test_invalid_arguments_return_status(sk):
     s = torch.cuda.current_stream().cuda_stream
     nbytes = ws.numel()
 
-    def call(B=1, H_q=8, H_kv=4, d=128, w=4, grid=0, wsb=nbytes, dt=sk.BF16, p=common):
+    def call(B=1, H_q=8, H_kv=4, d=128, w=4, grid=0, wsb=nbytes, dt=sk.BF16, p=common, fl=0):
         return lib.speechkv_decode_attn(*p, B, H_q, H_kv, d, w, 0, 0, grid, ws.data_ptr(), wsb,
-                                        dt, s)
+                                        dt, fl, s)
     assert call() == sk.OK
     assert call(w=0) == sk.ERR_INVALID_ARG
     assert call(H_q=7) == sk.ERR_INVALID_ARG
@@ -275,6 +275,8 @@ def test_invalid_arguments_return_status(sk):
     assert call(B=sk.MAX_BATCH + 1) == sk.ERR_UNSUPPORTED
     assert call(wsb=16) == sk.ERR_WORKSPACE
     assert call(grid=-1) == sk.ERR_INVALID_ARG
+    assert call(fl=2) == sk.ERR_INVALID_ARG                   # unknown flag
+    assert call(fl=sk.OVERLAP_PRIOR) == sk.OK
     misaligned = (q.data_ptr() + 2,) + common[1:]
     assert call(p=misaligned) == sk.ERR_INVALID_ARG
     nullq = (None,) + common[1:]
@@ -365,6 +367,55 @@ def test_fused_step_matches_separate_calls_and_writes_cache(sk):
         assert torch.equal(A.k, Bc.k) and torch.equal(A.v, Bc.v)
         H.assert_close(H.f64(outB), H.f64(outA), "bf16", f"step {step}")
     assert sk.check_device_error() == sk.OK
+
+
+@pytest.mark.parametrize("graph", [False, True])
+def test_overlap_prior_interleaved_layers(sk, oracle, graph):
+    """SPEECHKV_OVERLAP_PRIOR between the decode steps of different layers
+    (the previous kernel writes another layer's cache, its length and the
+    shared workspace): results still match the oracle, eagerly and when the
+    steps are captured in a CUDA graph."""
+    wl = inputs.qwen_ragged(B=5)
+    layers, steps = [wl.l0 - 1, wl.l0, wl.l0 + 1], 3
+    gl, ol = [], []
+    for layer in layers:
+        L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=steps)
+        gl.append(L)
+        ol.append(H.oracle_prefill(oracle, wl, layer, steps, ks, vs, gate))
+    ws = _ws(sk, wl)
+    ins = [[[x.cuda() for x in inputs.step_qkv(wl, layer, t)] for layer in layers]
+           for t in range(steps)]
+    outs = [[torch.empty_like(ins[0][0][0]) for _ in layers] for _ in range(steps)]
+
+    def run():
+        for t in range(steps):
+            for i, layer in enumerate(layers):
+                q, kn, vn = ins[t][i]
+                L = gl[i]
+                sk.decode_step(q, kn, vn, L.k, L.v, L.cache_off, L.len, outs[t][i], ws, wl.w,
+                               layer, wl.l0, flags=sk.OVERLAP_PRIOR)
+    if graph:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            run()
+        g.replay()
+    else:
+        run()
+    torch.cuda.synchronize()
+    assert sk.check_device_error() == sk.OK
+    for t in range(steps):
+        for i, layer in enumerate(layers):
+            q, kn, vn = (x.cpu() for x in ins[t][i])
+            ref = []
+            for b in range(wl.B):
+                Kc, Vc, n = ol[i][b]
+                n = oracle.append_request(Kc, Vc, n, H.f64(kn[b]), H.f64(vn[b]))
+                ol[i][b][2] = n
+                ref.append(oracle.decode_attn_request(H.f64(q[b]), Kc[:n], Vc[:n],
+                                                      storage=oracle.STORE_BF16))
+            H.assert_close(H.f64(outs[t][i]), np.stack(ref), "bf16", f"step {t} layer {layer}")
+    for i in range(len(layers)):
+        assert [int(x) for x in gl[i].len.cpu()] == [o[2] for o in ol[i]]
 
 
 def test_fused_step_full_cache(sk, oracle):
