@@ -157,7 +157,8 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     // before touching anything.  With overlap, the prologue and the bulk
     // copies of cached rows run first; every read of q / k_new / v_new and
     // every global write (outputs, cache rows, len, workspace) comes after
-    // griddep_wait(), and every thread waits before it exits.
+    // griddep_wait(), and every warp but the producer's idle lanes waits
+    // before it exits (so this grid never completes before the previous one).
     griddep_launch_dependents();
     if (!overlap) griddep_wait();
 
@@ -220,7 +221,11 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int64_t U = (int64_t)H_kv * cum[B];
     const int64_t Cn = U < (int64_t)gridDim.x ? U : (int64_t)gridDim.x;
     const int64_t c = blockIdx.x;
-    if (warp == W + 1) {
+    // Work that reads what the previous kernel may produce (k_new, v_new) or
+    // writes global memory waits for it.  The producer is the first warp to
+    // wait (after its first copies); the others do this part only once the
+    // first tile -- whose queries are copied after that wait -- has landed.
+    auto merge_warp_prior_part = [&]() {  // merge warp
         griddep_wait();
         // empty requests get a zero output (softmax over nothing)
         for (int b = blockIdx.x; b < B; b += gridDim.x) {
@@ -228,53 +233,61 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             for (int i = lane; i < H_q * D; i += 32)
                 out[(int64_t)b * H_q * D + i] = from_float<T>(0.f);
         }
-    }
-    if (kAppend && warp == W + 1) {
-        // every CTA has read len[] once past the prologue's barrier; the last
-        // one to get here advances len[] of the requests that took a token
-        int last = 0;
-        if (lane == 0) last = atomic_add_acq_rel_gpu(done, 1) == (int)gridDim.x - 1;
-        last = __shfl_sync(0xffffffffu, last, 0);
-        __syncwarp();
-        if (last) {
-            for (int b = lane; b < B; b += 32)
-                if (newrow[b] >= 0) len[b] = newrow[b] + 1;
+        if (kAppend) {
+            // every CTA has read len[] before its prologue barrier; the last
+            // one to get here advances len[] of the requests that took a token
+            int last = 0;
+            if (lane == 0) last = atomic_add_acq_rel_gpu(done, 1) == (int)gridDim.x - 1;
+            last = __shfl_sync(0xffffffffu, last, 0);
             __syncwarp();
-            if (lane == 0) *done = 0;
-        }
-    }
-    if (kAppend && warp < W) {
-        griddep_wait();
-        // write the new tokens into their cache rows (nothing in this kernel
-        // reads those rows from the cache: the new row comes from k_new/v_new)
-        constexpr int kVec = 16 / (int)sizeof(T);
-        const int nvec = H_kv * D / kVec;  // 16-byte vectors per token
-        for (int b = blockIdx.x; b < B; b += gridDim.x) {
-            const int32_t nr = newrow[b];
-            if (nr < 0) continue;
-            const int64_t cap = offs[b + 1] - offs[b];
-            for (int i = tid; i < 2 * nvec; i += W * 32) {
-                const int tensor = i >= nvec;
-                const int e = (i - tensor * nvec) * kVec;
-                const int hh = e / D, col = e - hh * D;
-                const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
-                T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D + col;
-                copy_bytes<16>(dst, src);
+            if (last) {
+                for (int b = lane; b < B; b += 32)
+                    if (newrow[b] >= 0) len[b] = newrow[b] + 1;
+                __syncwarp();
+                if (lane == 0) *done = 0;
             }
         }
-    }
-    if (c >= Cn) {
+    };
+    auto consumer_prior_part = [&]() {  // consumer warps
         griddep_wait();
+        if (kAppend) {
+            // write the new tokens into their cache rows (nothing in this
+            // kernel reads those rows from the cache: the attention takes the
+            // new row from k_new / v_new)
+            constexpr int kVec = 16 / (int)sizeof(T);
+            const int nvec = H_kv * D / kVec;  // 16-byte vectors per token
+            for (int b = blockIdx.x; b < B; b += gridDim.x) {
+                const int32_t nr = newrow[b];
+                if (nr < 0) continue;
+                const int64_t cap = offs[b + 1] - offs[b];
+                for (int i = tid; i < 2 * nvec; i += W * 32) {
+                    const int tensor = i >= nvec;
+                    const int e = (i - tensor * nvec) * kVec;
+                    const int hh = e / D, col = e - hh * D;
+                    const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
+                    T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D +
+                             col;
+                    copy_bytes<16>(dst, src);
+                }
+            }
+        }
+    };
+    if (c >= Cn) {  // no rows for this CTA
+        if (warp == W + 1)
+            merge_warp_prior_part();
+        else if (warp < W)
+            consumer_prior_part();
+        else
+            griddep_wait();
         return;
     }
     const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
 
     if (warp == W) {
         // ================= producer: one lane issues bulk copies ============
-        if (lane != 0) {
-            griddep_wait();
-            return;
-        }
+        // lanes 1..31 leave at once: a grid dependency wait on this warp would
+        // also hold lane 0 back (the other warps' waits order the CTA's exit)
+        if (lane != 0) return;
         int stage = 0;
         uint32_t phase = 0;
         int64_t issued = 0;
@@ -374,6 +387,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             const uint32_t use = (uint32_t)((k >> 1) & 1);
             bool ok = !flags[0] && mbar_wait_bounded(&piece_bar[x], use, err);
             ok = __all_sync(0xffffffffu, ok) && !__shfl_sync(0xffffffffu, flags[0], 0);
+            if (k == 0) merge_warp_prior_part();
             const float *mo = mrg + x * C::kMergeFloats;  // [W][G][D]
             const float *mm = mo + W * G * D;              // [W][G]
             const float *ml = mm + W * G;                  // [W][G]
@@ -497,6 +511,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     int stage = 0;
     uint32_t phase = 0;
     bool aborted = false;
+    bool prior_part_done = false;
     int64_t k = 0;  // piece index within this CTA
     for (int64_t u = u0; u < u1; k++) {
         const Piece p = piece_at(cum, B, H_kv, u, u1);
@@ -522,6 +537,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                     flags[0] = 1;
                     aborted = true;
                 }
+            }
+            if (!prior_part_done) {
+                consumer_prior_part();
+                prior_part_done = true;
             }
             const unsigned char *ks = stages + (size_t)stage * C::kStageBytes;
             if (!aborted && t == p.t0) {
@@ -665,6 +684,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         if (lane == 0) mbar_arrive(&piece_bar[x]);
         u += p.t1 - p.t0;
     }
+    if (!prior_part_done) consumer_prior_part();  // (only if there was no tile)
     griddep_wait();
 }
 
