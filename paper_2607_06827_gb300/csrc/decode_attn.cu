@@ -64,7 +64,9 @@ struct DecodeCfg {
     static constexpr int kMergeFloats = kWarps * G * D + 2 * kWarps * G;
     static constexpr int kMergeBytes = 2 * kMergeFloats * 4;
     static constexpr int kBarBytes = (2 * 3 + 4) * 8;  // full/empty per stage (<= 3), piece/free x2
-    static constexpr int kSmemLimit = 227 * 1024;
+    // shared memory per CTA: an SM has 228 KB, of which 1 KB per resident CTA
+    // is reserved
+    static constexpr int kSmemLimit = 228 * 1024 / kCtasPerSm - 1024;
     // per-request tables: prefix sums of rows and cache offsets (int64, B+1
     // each) and the row an appended token takes (int32, B, padded)
     static size_t table_bytes(int B) { return (size_t)(B + 1) * 16 + ((size_t)B * 4 + 15) / 16 * 16; }
