@@ -240,6 +240,38 @@ speechkv_status speechkv_decode_step(const void *q, const void *k_new,
                                      cudaStream_t stream);
 
 /*
+ * speechkv_decode_step_noalloc -- speechkv_decode_step for callers that
+ * cannot allocate device memory.  The paper has no counterpart: this entry
+ * point only changes where the split-K scratch lives.
+ *
+ * Some callers may not allocate GPU memory at all: a plug-in running inside
+ * a serving process whose memory pool owns every byte of the device, or a
+ * latency-critical path that must never enter an allocator (whose calls can
+ * block, synchronise the device or fail).  Such a caller passes no
+ * workspace: the scratch is a fixed array of SPEECHKV_NOALLOC_SCRATCH_BYTES
+ * in device memory that the library itself owns (every GPU that loads the
+ * library holds it until the process exits).  This call allocates nothing.
+ *
+ * Arguments, results and errors are those of speechkv_decode_step, minus the
+ * workspace.  A batch whose scratch (speechkv_decode_workspace_size for the
+ * same shapes and grid) exceeds SPEECHKV_NOALLOC_SCRATCH_BYTES is refused with
+ * SPEECHKV_ERR_WORKSPACE before anything runs.  The first call on a device
+ * looks up the array's device address (a one-time set-up per device); make
+ * that first call before any stream capture.  Every call shares the one
+ * array, which keeps the previous call's contents: each call zeroes the
+ * counters it needs on `stream` before launching, and calls that may run at
+ * the same time on one device (for example on two streams) race on it.
+ */
+#define SPEECHKV_NOALLOC_SCRATCH_BYTES (8u << 20)
+
+speechkv_status speechkv_decode_step_noalloc(
+    const void *q, const void *k_new, const void *v_new, void *k_cache,
+    void *v_cache, const int64_t *cache_off, int32_t *len, void *out,
+    float scale, int32_t B, int32_t H_q, int32_t H_kv, int32_t d, int32_t w,
+    int32_t layer, int32_t l0, int32_t grid_ctas, speechkv_dtype dtype,
+    uint32_t flags, cudaStream_t stream);
+
+/*
  * Synchronises `stream`, then reads and clears the current device's error
  * word.  Returns SPEECHKV_OK when no kernel reported an error since the last
  * check, else the first error reported (CAPACITY, INVALID_ARG or TIMEOUT),

@@ -320,3 +320,68 @@ speechkv_status speechkv_check_device_error(cudaStream_t stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of speechkv_decode_step (no counterpart in the
+// paper).  Its split-K scratch lives in a fixed-size array in device memory
+// that belongs to the library itself, so the caller passes no workspace.
+// ---------------------------------------------------------------------------
+
+// Every GPU that loads this library holds this array until the process exits.
+static __device__ __align__(256) unsigned char speechkv_noalloc_scratch[SPEECHKV_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+void *g_noalloc_scratch[kMaxDevices];  // the array's device address, per device
+
+// In host code `speechkv_noalloc_scratch` names a host-side stand-in, not the
+// device memory; kernels must be given the address cudaGetSymbolAddress
+// returns for the current device.  Done once per device, on first use.
+speechkv_status noalloc_scratch(void **out) {
+    int dev = 0;
+    speechkv_status st = current_device(&dev);
+    if (st != SPEECHKV_OK) return st;
+    std::lock_guard<std::mutex> lock(g_mu);
+    if (!g_noalloc_scratch[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, speechkv_noalloc_scratch) != cudaSuccess || !p)
+            return SPEECHKV_ERR_CUDA;
+        g_noalloc_scratch[dev] = p;
+    }
+    *out = g_noalloc_scratch[dev];
+    return SPEECHKV_OK;
+}
+
+}  // namespace
+
+extern "C" speechkv_status speechkv_decode_step_noalloc(
+    const void *q, const void *k_new, const void *v_new, void *k_cache, void *v_cache,
+    const int64_t *cache_off, int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+    int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0, int32_t grid_ctas,
+    speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
+    if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || grid_ctas < 0)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    void *scratch = nullptr;
+    st = noalloc_scratch(&scratch);
+    if (st != SPEECHKV_OK) return st;
+    int grid = grid_ctas;
+    if (grid == 0) {
+        st = decode_auto_grid(s, dtype, d, H_q / H_kv, B, &grid);
+        if (st != SPEECHKV_OK) return st;
+    }
+    // a batch whose scratch would not fit is refused before anything runs
+    if (workspace_bytes(B, H_q, H_kv, d, grid) > (size_t)SPEECHKV_NOALLOC_SCRATCH_BYTES)
+        return SPEECHKV_ERR_WORKSPACE;
+    // the counters must start at zero; the array keeps the previous call's data
+    if (cudaMemsetAsync(scratch, 0, counters_bytes(B, H_kv), stream) != cudaSuccess)
+        return SPEECHKV_ERR_CUDA;
+    return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
+                         H_kv, d, w, layer, l0, grid, scratch, SPEECHKV_NOALLOC_SCRATCH_BYTES,
+                         dtype, flags, stream, true);
+}

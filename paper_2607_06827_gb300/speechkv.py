@@ -42,6 +42,10 @@ SIGNATURES = {
                                             _I32, _I32, _I32, _I32, _I32, _I32,
                                             _I32, _I32, _P, _SZ, ctypes.c_int,
                                             ctypes.c_uint32, _P]),
+    "speechkv_decode_step_noalloc": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _F,
+                                                    _I32, _I32, _I32, _I32, _I32, _I32,
+                                                    _I32, _I32, ctypes.c_int,
+                                                    ctypes.c_uint32, _P]),
     "speechkv_check_device_error": (ctypes.c_int, [_P]),
 }
 
@@ -173,6 +177,21 @@ def decode_step(q, k_new, v_new, k_cache, v_cache, cache_off, length, out, works
         _ptr(workspace), workspace.numel() * workspace.element_size(), _dtype_code(q), flags,
         _stream(stream)),
         "speechkv_decode_step")
+
+
+def decode_step_noalloc(q, k_new, v_new, k_cache, v_cache, cache_off, length, out, w: int,
+                        layer: int, l0: int, scale: float = 0.0, grid_ctas: int = 0,
+                        flags: int = 0, stream=None):
+    """speechkv_decode_step_noalloc: decode_step for callers that may not
+    allocate device memory; the library's own fixed scratch replaces the
+    workspace (see include/speechkv.h for its size limit and sharing rules)."""
+    B, H_q, d = q.shape
+    H_kv = k_new.shape[1]
+    _check(load().speechkv_decode_step_noalloc(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache), _ptr(v_cache), _ptr(cache_off),
+        _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas,
+        _dtype_code(q), flags, _stream(stream)),
+        "speechkv_decode_step_noalloc")
 
 
 def check_device_error(stream=None) -> int:
