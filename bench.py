@@ -569,9 +569,12 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(bytes_per_launch_all: float):
-    """DRAM bytes per decode_attn launch from the committed ncu summary, if it
-    was taken on the current kernel source; else None."""
+def profiled_traffic(bytes_per_launch: float):
+    """DRAM bytes per decode-attention launch of this workload, from the
+    committed ncu capture (one pooled layer), scaled by the rows processed:
+    captured traffic x (this workload's algorithmic bytes per launch / the
+    captured launch's algorithmic bytes).  None when the capture was taken on
+    another kernel source."""
     try:
         kv = {}
         with open(PROFILE_TRAFFIC) as f:
@@ -581,8 +584,9 @@ def profiled_traffic(bytes_per_launch_all: float):
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_sha256_16") != kernel_hash():
             return None
-        return float(kv["dram_bytes_per_launch"])
-    except (OSError, ValueError, KeyError):
+        scale = bytes_per_launch / float(kv["algorithmic_bytes"])
+        return round(float(kv["dram_bytes_per_launch"]) * scale)
+    except (OSError, ValueError, KeyError, ZeroDivisionError):
         return None
 
 
