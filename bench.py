@@ -81,32 +81,43 @@ def parse_args():
 # distributed plumbing (replicas only: no data-path collective)
 # ---------------------------------------------------------------------------
 class Dist:
-    def __init__(self, n_gpus: int):
+    """Replica bookkeeping for N GPUs: rank/world from the torchrun
+    environment, a barrier and the max of the timings over ranks.  NCCL on
+    GPUs; gloo when CUDA is absent (the CPU tests of this logic).  There is no
+    data-path collective: every rank runs its own batch."""
+
+    def __init__(self, n_gpus: int = 1, backend: str | None = None):
         import torch
         self.world = int(os.environ.get("WORLD_SIZE", "1"))
         self.rank = int(os.environ.get("RANK", "0"))
         self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.cuda = torch.cuda.is_available()
         self.pg = None
         if self.world > 1:
             import torch.distributed as dist
-            torch.cuda.set_device(self.local)
-            dist.init_process_group("nccl")
+            if self.cuda:
+                torch.cuda.set_device(self.local)
+            dist.init_process_group(backend or ("nccl" if self.cuda else "gloo"))
             self.pg = dist
-        elif torch.cuda.is_available():
+        elif self.cuda:
             torch.cuda.set_device(0)
 
+    def _sync(self):
+        if self.cuda:
+            import torch
+            torch.cuda.synchronize()
+
     def barrier(self):
-        import torch
-        torch.cuda.synchronize()
+        self._sync()
         if self.pg:
             self.pg.barrier()
-        torch.cuda.synchronize()
+        self._sync()
 
     def max(self, x: float) -> float:
         if not self.pg:
             return x
         import torch
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        t = torch.tensor([x], dtype=torch.float64, device="cuda" if self.cuda else "cpu")
         self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
         return float(t.item())
 
