@@ -2,17 +2,19 @@
 // and layer at prefill (Sec. III-C) -- writes the compressed cache rows of
 // every (request, KV head) from the full-resolution prefill keys/values.
 //
-// One warp produces one cached row of one (request, KV head).  Task
-// tau = r * H_kv + h enumerates (prefill row r, head h); the request b holding
-// r is found by binary search over full_off, and t = r - full_off[b] is used
-// as the OUTPUT row index, so the first len_b tasks of a request are busy and
-// the rest idle.  Consecutive warps handle the heads of one token, which read
-// one contiguous token-major prefill row between them.
+// Grid (X, B): the X CTAs of request b share its output rows.  A warp task is
+// (output row t, chunk of heads): one chunk is at most 2 KB of a token-major
+// prefill row (8 heads of d = 128 in bf16), read with 16-byte loads that
+// cover 512 contiguous bytes per warp instruction.  Each 16-byte vector
+// belongs to one head, and the vectors of a head sit on consecutive lanes,
+// so a head's gate logit u_h . k_j is a shuffle reduction over those lanes
+// (deterministic order).
 //
 //   t <  P            text before the speech: copy prefill row t
 //   t <  P + n        speech window i = t - P: online softmax over the gate
-//                     logits u_h . k_j of frames P + i*w .. min(.., P + T) - 1,
-//                     weighted sums of keys and values (fp32), one rounding
+//                     logits of frames P + i*w .. min(.., P + T) - 1 (up to 4
+//                     frames in flight), weighted sums of keys and values in
+//                     fp32, one rounding to the storage type
 //   t <  P + n + N    text after the speech: copy prefill row t - n + T
 //
 // With w_eff = 1 (layers before l0) every row is a bit-exact copy.
@@ -24,157 +26,175 @@
 namespace speechkv {
 namespace {
 
-// Largest b with full_off[b] <= r, for r < full_off[B].
-__device__ __forceinline__ int request_of_row(const int64_t *__restrict__ off, int B, int64_t r) {
-    int lo = 0, hi = B - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (__ldg(off + mid) <= r)
-            lo = mid;
-        else
-            hi = mid - 1;
-    }
-    return lo;
-}
+constexpr int kPoolWarps = 8;
+constexpr int kPoolFrames = 4;  // frames of a window loaded at once
 
 template <typename T, int D>
-__global__ void __launch_bounds__(256)
+struct PoolCfg {
+    static constexpr int kEpv = 16 / (int)sizeof(T);             // elements per 16-byte vector
+    static constexpr int kVecPerHead = D * (int)sizeof(T) / 16;  // 8, 16 or 32
+    static constexpr int kHeadsPerChunk = 2048 / (D * (int)sizeof(T));
+    static constexpr int kVpl = kHeadsPerChunk * kVecPerHead / 32;  // vectors per lane
+    static_assert(kVecPerHead <= 32 && 32 % kVecPerHead == 0, "head layout");
+    static_assert(kVpl >= 1 && kVpl * 32 * 16 == 2048, "chunk layout");
+};
+
+template <typename T, int D>
+__global__ void __launch_bounds__(kPoolWarps * 32)
     pool_kernel(const T *__restrict__ kf, const T *__restrict__ vf,
                 const int64_t *__restrict__ full_off, const int32_t *__restrict__ Pa,
                 const int32_t *__restrict__ Ta, const int32_t *__restrict__ Na,
                 const float *__restrict__ gate, T *__restrict__ kc, T *__restrict__ vc,
-                const int64_t *__restrict__ cache_off, int32_t *__restrict__ len, int B,
+                const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
                 int64_t full_rows, int H_kv, int w, int *__restrict__ err) {
-    constexpr int kCols = D / 32;  // elements per lane
-    const int lane = threadIdx.x & 31;
-    const int64_t gwarp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    using C = PoolCfg<T, D>;
+    constexpr int VPL = C::kVpl, EPV = C::kEpv, VH = C::kVecPerHead;
+    const int b = blockIdx.y;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-    // lengths: the first B threads of the grid
-    const int64_t gtid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (gtid < B) {
-        const int b = (int)gtid;
-        const int64_t S = full_off[b + 1] - full_off[b];
-        const int64_t cap = cache_off[b + 1] - cache_off[b];
-        const int64_t Pb = Pa[b], Tb = Ta[b], Nb = Na[b];
-        const int64_t n = (Tb + w - 1) / w;
-        int64_t L = Pb + n + Nb;
-        if (Pb < 0 || Tb < 0 || Nb < 0 || S != Pb + Tb + Nb || cap < 0 || full_off[b] < 0 ||
-            full_off[b + 1] > full_rows || cache_off[b] < 0) {
+    const int64_t row0 = full_off[b], S = full_off[b + 1] - row0;
+    const int64_t base = cache_off[b], cap = cache_off[b + 1] - base;
+    const int64_t Pb = Pa[b], Tb = Ta[b], Nb = Na[b];
+    const int64_t n = (Tb + w - 1) / w;
+    const int64_t L = Pb + n + Nb;
+    const bool bad = Pb < 0 || Tb < 0 || Nb < 0 || S != Pb + Tb + Nb || cap < 0 || row0 < 0 ||
+                     full_off[b + 1] > full_rows || base < 0;
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        if (bad)
             report_error(err, SPEECHKV_ERR_INVALID_ARG);
-            L = 0;
-        } else if (L > cap) {
+        else if (L > cap)
             report_error(err, SPEECHKV_ERR_CAPACITY);
-            L = cap;
-        }
-        len[b] = (int32_t)L;
+        len[b] = (int32_t)(bad ? 0 : (L < cap ? L : cap));
     }
+    if (bad) return;
+    const int64_t rows_out = L < cap ? L : cap;  // rows beyond the capacity are not written
 
-    const int64_t tasks = full_rows * H_kv;
-    for (int64_t tau = gwarp; tau < tasks; tau += nwarps) {
-        const int64_t r = tau / H_kv;
-        const int h = (int)(tau - r * H_kv);
-        if (r >= __ldg(full_off + B) || r < __ldg(full_off)) continue;
-        const int b = request_of_row(full_off, B, r);
-        const int64_t row0 = __ldg(full_off + b);
-        const int64_t t = r - row0;
-        const int64_t Pb = __ldg(Pa + b), Tb = __ldg(Ta + b), Nb = __ldg(Na + b);
-        const int64_t S = __ldg(full_off + b + 1) - row0;
-        if (Pb < 0 || Tb < 0 || Nb < 0 || S != Pb + Tb + Nb || row0 < 0 ||
-            __ldg(full_off + b + 1) > full_rows || __ldg(cache_off + b) < 0)
-            continue;  // reported above
-        const int64_t n = (Tb + w - 1) / w;
-        if (t >= Pb + n + Nb) continue;  // idle task
-        const int64_t cap = __ldg(cache_off + b + 1) - __ldg(cache_off + b);
-        if (t >= cap) continue;        // reported above (capacity)
-        T *kd = kc + ((__ldg(cache_off + b) * H_kv + (int64_t)h * cap + t) * D) + lane * kCols;
-        T *vd = vc + ((__ldg(cache_off + b) * H_kv + (int64_t)h * cap + t) * D) + lane * kCols;
-        const int64_t rowstride = (int64_t)H_kv * D;
-        const T *kbase = kf + (row0 * H_kv + h) * D + lane * kCols;  // prefill row 0 of b
-        const T *vbase = vf + (row0 * H_kv + h) * D + lane * kCols;
+    const int nchunk = (H_kv + C::kHeadsPerChunk - 1) / C::kHeadsPerChunk;
+    const int64_t tasks = rows_out * nchunk;
+    const int64_t rowstride = (int64_t)H_kv * D;  // elements per prefill row
+    for (int64_t task = (int64_t)blockIdx.x * kPoolWarps + warp; task < tasks;
+         task += (int64_t)gridDim.x * kPoolWarps) {
+        const int64_t t = task / nchunk;
+        const int h0 = (int)(task - t * nchunk) * C::kHeadsPerChunk;
+        const int hc = H_kv - h0 < C::kHeadsPerChunk ? H_kv - h0 : C::kHeadsPerChunk;
+        const int nv = hc * VH;  // vectors of this chunk
+        // the lane's vectors: v = lane + 32 i, of head h0 + v / VH
+        bool act[VPL];
+        int hv[VPL], cv[VPL];
+#pragma unroll
+        for (int i = 0; i < VPL; i++) {
+            const int v = lane + 32 * i;
+            act[i] = v < nv;
+            hv[i] = h0 + v / VH;
+            cv[i] = (v % VH) * EPV;
+        }
+        auto dst_of = [&](T *cache, int i) {
+            return cache + (base * H_kv + (int64_t)hv[i] * cap + t) * D + cv[i];
+        };
+        // prefill row 0 of request b, this lane's first vector of the chunk
+        const T *kb = kf + row0 * rowstride + (int64_t)h0 * D + lane * EPV;
+        const T *vb = vf + row0 * rowstride + (int64_t)h0 * D + lane * EPV;
 
         if (t < Pb || t >= Pb + n || w == 1) {
+            // text row (or no pooling): bit-exact copy
             const int64_t src = (t < Pb || w == 1) ? t : t - n + Tb;
-            copy_bytes<kCols * (int)sizeof(T)>(kd, kbase + src * rowstride);
-            copy_bytes<kCols * (int)sizeof(T)>(vd, vbase + src * rowstride);
+#pragma unroll
+            for (int i = 0; i < VPL; i++) {
+                if (!act[i]) continue;
+                copy_bytes<16>(dst_of(kc, i), kb + src * rowstride + 32 * i * EPV);
+                copy_bytes<16>(dst_of(vc, i), vb + src * rowstride + 32 * i * EPV);
+            }
             continue;
         }
 
         // pooled speech row: frames [j0, j1) of the prefill rows
-        const int64_t i = t - Pb;
-        const int64_t j0 = Pb + i * w;
+        const int64_t j0 = Pb + (t - Pb) * w;
         const int64_t j1 = (j0 + w < Pb + Tb) ? j0 + w : Pb + Tb;
-        float u[kCols];
+        float u[VPL][EPV];
 #pragma unroll
-        for (int c = 0; c < kCols; c++) u[c] = __ldg(gate + h * D + lane * kCols + c);
-        float mx = -INFINITY, sum = 0.f, ak[kCols], av[kCols];
+        for (int i = 0; i < VPL; i++)
 #pragma unroll
-        for (int c = 0; c < kCols; c++) ak[c] = av[c] = 0.f;
-        for (int64_t j = j0; j < j1; j += 4) {
-            // four frames in flight, then their logits and the online update
-            float kx[4][kCols], vx[4][kCols], z[4];
+            for (int e = 0; e < EPV; e++)
+                u[i][e] = act[i] ? __ldg(gate + hv[i] * D + cv[i] + e) : 0.f;
+        float mx[VPL], sum[VPL], ak[VPL][EPV], av[VPL][EPV];
 #pragma unroll
-            for (int f = 0; f < 4; f++) {
-                if (j + f < j1) {
-                    load_vec<T, kCols>(kbase + (j + f) * rowstride, kx[f]);
-                    load_vec<T, kCols>(vbase + (j + f) * rowstride, vx[f]);
+        for (int i = 0; i < VPL; i++) {
+            mx[i] = -INFINITY;
+            sum[i] = 0.f;
+#pragma unroll
+            for (int e = 0; e < EPV; e++) ak[i][e] = av[i][e] = 0.f;
+        }
+        for (int64_t j = j0; j < j1; j += kPoolFrames) {
+            float kx[kPoolFrames][VPL][EPV], vx[kPoolFrames][VPL][EPV];
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++)
+#pragma unroll
+                for (int i = 0; i < VPL; i++) {
+                    if (j + f < j1 && act[i]) {
+                        load_vec<T, EPV>(kb + (j + f) * rowstride + 32 * i * EPV, kx[f][i]);
+                        load_vec<T, EPV>(vb + (j + f) * rowstride + 32 * i * EPV, vx[f][i]);
+                    } else {
+#pragma unroll
+                        for (int e = 0; e < EPV; e++) kx[f][i][e] = vx[f][i][e] = 0.f;
+                    }
                 }
-            }
 #pragma unroll
-            for (int f = 0; f < 4; f++) {
-                float s = 0.f;
-                if (j + f < j1) {
-#pragma unroll
-                    for (int c = 0; c < kCols; c++) s = fmaf(u[c], kx[f][c], s);
-                }
-                z[f] = warp_sum(s);
-            }
-#pragma unroll
-            for (int f = 0; f < 4; f++) {
+            for (int f = 0; f < kPoolFrames; f++) {
                 if (j + f >= j1) break;
-                const float mnew = fmaxf(mx, z[f]);
-                const float corr = expf(mx - mnew);  // 0 on the first frame
-                const float e = expf(z[f] - mnew);
-                sum = sum * corr + e;
 #pragma unroll
-                for (int c = 0; c < kCols; c++) {
-                    ak[c] = fmaf(e, kx[f][c], ak[c] * corr);
-                    av[c] = fmaf(e, vx[f][c], av[c] * corr);
+                for (int i = 0; i < VPL; i++) {
+                    // logit of this vector's head: reduce over its VH lanes
+                    float z = 0.f;
+#pragma unroll
+                    for (int e = 0; e < EPV; e++) z = fmaf(u[i][e], kx[f][i][e], z);
+#pragma unroll
+                    for (int o = 1; o < VH; o <<= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+                    const float mnew = fmaxf(mx[i], z);
+                    const float corr = expf(mx[i] - mnew);  // 0 on the first frame
+                    const float p = expf(z - mnew);
+                    sum[i] = sum[i] * corr + p;
+#pragma unroll
+                    for (int e = 0; e < EPV; e++) {
+                        ak[i][e] = fmaf(p, kx[f][i][e], ak[i][e] * corr);
+                        av[i][e] = fmaf(p, vx[f][i][e], av[i][e] * corr);
+                    }
+                    mx[i] = mnew;
                 }
-                mx = mnew;
             }
         }
-        const float inv = 1.f / sum;
 #pragma unroll
-        for (int c = 0; c < kCols; c++) {
-            ak[c] *= inv;
-            av[c] *= inv;
+        for (int i = 0; i < VPL; i++) {
+            if (!act[i]) continue;
+            const float inv = 1.f / sum[i];
+#pragma unroll
+            for (int e = 0; e < EPV; e++) {
+                ak[i][e] *= inv;
+                av[i][e] *= inv;
+            }
+            store_vec<T, EPV>(dst_of(kc, i), ak[i]);
+            store_vec<T, EPV>(dst_of(vc, i), av[i]);
         }
-        store_vec<T, kCols>(kd, ak);
-        store_vec<T, kCols>(vd, av);
     }
 }
 
 template <typename T, int D>
 cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t stream) {
-    const int64_t tasks = a.full_rows * a.H_kv;
-    const int64_t warps_per_block = 8;
-    int64_t blocks = (tasks + warps_per_block - 1) / warps_per_block;
-    const int64_t bmin = (a.B + 255) / 256;  // the length writers
-    if (blocks < bmin) blocks = bmin;
-    const int64_t cap = (int64_t)num_sms * 16;  // grid-stride beyond this
-    if (blocks > cap) blocks = cap;
-    if (blocks < 1) blocks = 1;
-    pool_kernel<T, D><<<(unsigned)blocks, 256, 0, stream>>>(
+    // about four CTAs per SM over the whole batch, at least one per request
+    int x = (4 * num_sms + a.B - 1) / a.B;
+    if (x < 1) x = 1;
+    if (x > 65535) x = 65535;
+    const dim3 grid((unsigned)x, (unsigned)a.B);
+    pool_kernel<T, D><<<grid, kPoolWarps * 32, 0, stream>>>(
         static_cast<const T *>(a.k_full), static_cast<const T *>(a.v_full), a.full_off, a.P, a.T,
         a.N, a.gate, static_cast<T *>(a.k_cache), static_cast<T *>(a.v_cache), a.cache_off,
-        a.len, a.B, a.full_rows, a.H_kv, a.w_eff, a.err);
+        a.len, a.full_rows, a.H_kv, a.w_eff, a.err);
     return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_pool(const PoolArgs &a, int num_sms, cudaStream_t stream) {
+    if (a.B > 65535) return cudaErrorInvalidValue;  // grid.y limit
     if (a.dtype == SPEECHKV_F32) {
         if (a.d == 64) return launch_pool_instance<float, 64>(a, num_sms, stream);
         if (a.d == 128) return launch_pool_instance<float, 128>(a, num_sms, stream);
