@@ -201,7 +201,7 @@ class DecodeModel:
         P, T, N = t32(wl.P), t32(wl.T), t32(wl.N)
         full_off_t = torch.tensor(full_off, dtype=torch.int64, device=device)
         self.k, self.v, self.len, self.off, self.rows0 = [], [], [], [], []
-        self.pool_ms = {}
+        self.pool_ms, self.pool_bytes = {}, {}
         for layer in self.layers:
             cap = [sk.compressed_len(wl.P[b], wl.T[b], wl.N[b], wl.G[b], wl.w, layer, wl.l0)
                    + steps_total for b in range(B)]
@@ -217,12 +217,18 @@ class DecodeModel:
             vf = inputs.device_normal((full_rows, Hk, d), self.dtype, device, wl.seed, seed_key, 2, layer)
             gate = inputs.device_normal((Hk, d), torch.float32, device, wl.seed, seed_key, 3, layer)
             gate /= math.sqrt(d)
+            # speechkv_pool is idempotent: the first call loads the kernel and
+            # leaves the cache (not the prefill rows) in L2; the second is timed
+            sk.pool(kf, vf, full_off_t, P, T, N, gate, kc, vc, offt, ln, wl.w, layer, wl.l0)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record()
             sk.pool(kf, vf, full_off_t, P, T, N, gate, kc, vc, offt, ln, wl.w, layer, wl.l0)
             e1.record()
             torch.cuda.synchronize()
             self.pool_ms[layer] = e0.elapsed_time(e1)
+            out_rows = sum(sk.compressed_len(wl.P[b], wl.T[b], wl.N[b], 0, wl.w, layer, wl.l0)
+                           for b in range(B))  # rows speechkv_pool writes
+            self.pool_bytes[layer] = (full_rows + out_rows) * Hk * d * 2 * 2  # K and V, bf16
             del kf, vf
             self.k.append(kc); self.v.append(vc); self.len.append(ln); self.off.append(offt)
         # tokens generated before the measured steps go through speechkv_append
@@ -370,6 +376,14 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
                                      len(comp) * 1e3 if comp else float("nan")),
         "pool_us_full_layer": (sum(model.pool_ms[model.layers[i]] for i in full) /
                                len(full) * 1e3 if full else float("nan")),
+        "pool_gbs_compressed_layer": (
+            sum(model.pool_bytes[model.layers[i]] for i in comp) /
+            (sum(model.pool_ms[model.layers[i]] for i in comp) * 1e-3) / 1e9
+            if comp else float("nan")),
+        "pool_gbs_full_layer": (
+            sum(model.pool_bytes[model.layers[i]] for i in full) /
+            (sum(model.pool_ms[model.layers[i]] for i in full) * 1e-3) / 1e9
+            if full else float("nan")),
         "gpu_launches": launches_a,
         "region_ms": ms_a,
     }

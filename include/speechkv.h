@@ -115,9 +115,9 @@ int64_t speechkv_compressed_len(int32_t P, int32_t T, int32_t N, int32_t G,
  *                 must hold exactly P[b] + T[b] + N[b] rows.
  * full_off        dev int64 [B+1], non-decreasing, full_off[B] <= full_rows.
  * P, T, N         dev int32 [B]: text before, speech frames, text after.
- * gate            dev fp32 [H_kv][d]: the gate vector u of g(k) = u . k for
- *                 this layer, one per KV head (no bias: a bias is constant
- *                 over a window and cancels in the softmax).
+ * gate            dev fp32 [H_kv][d], 16-byte aligned: the gate vector u of
+ *                 g(k) = u . k for this layer, one per KV head (no bias: a
+ *                 bias is constant over a window and cancels in the softmax).
  * k_cache,v_cache dev, this layer's cache blocks (layout above).
  * cache_off       dev int64 [B+1], capacities in rows.
  * len             dev int32 [B], written.

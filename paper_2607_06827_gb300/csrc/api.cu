@@ -209,7 +209,7 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full, const int6
     if (!aligned(k_full, 16) || !aligned(v_full, 16) || !aligned(k_cache, 16) ||
         !aligned(v_cache, 16) || !aligned(full_off, 8) || !aligned(cache_off, 8) ||
         !aligned(P, 4) || !aligned(T, 4) || !aligned(N, 4) || !aligned(len, 4) ||
-        !aligned(gate, 4))
+        !aligned(gate, 16))
         return SPEECHKV_ERR_INVALID_ARG;
     DeviceState *s = nullptr;
     speechkv_status st = device_state(&s);

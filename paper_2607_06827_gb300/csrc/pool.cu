@@ -2,22 +2,27 @@
 // and layer at prefill (Sec. III-C) -- writes the compressed cache rows of
 // every (request, KV head) from the full-resolution prefill keys/values.
 //
-// Grid (X, B): the X CTAs of request b share its output rows.  A warp task is
-// (output row t, chunk of heads): one chunk is at most 2 KB of a token-major
-// prefill row (8 heads of d = 128 in bf16), read with 16-byte loads that
-// cover 512 contiguous bytes per warp instruction.  Each 16-byte vector
-// belongs to one head, and the vectors of a head sit on consecutive lanes,
-// so a head's gate logit u_h . k_j is a shuffle reduction over those lanes
-// (deterministic order).
+// Grid (X, B): the X CTAs of request b share its output rows in two phases.
 //
-//   t <  P            text before the speech: copy prefill row t
-//   t <  P + n        speech window i = t - P: online softmax over the gate
-//                     logits of frames P + i*w .. min(.., P + T) - 1 (up to 4
-//                     frames in flight), weighted sums of keys and values in
-//                     fp32, one rounding to the storage type
-//   t <  P + n + N    text after the speech: copy prefill row t - n + T
+//   copy phase    rows kept unchanged -- text before the speech (t < P), text
+//                 after it (t >= P + n, prefill row t - n + T), or every row
+//                 when w_eff = 1 (layers before l0).  One flat index over
+//                 (row, 16-byte vector) for the whole CTA group; each thread
+//                 moves several independent vectors of K and V per iteration.
+//                 Bit-exact.
+//   pooled phase  speech window i (t = P + i): one warp per (window, chunk of
+//                 heads), one 16-byte vector of a head per lane, so a chunk is
+//                 512 contiguous bytes of a token-major prefill row.  The
+//                 gate logit u_h . k_j of a frame is a shuffle reduction over
+//                 the lanes of its head (fixed order); up to kPoolFrames
+//                 frames are loaded at once, their softmax weights taken in
+//                 base 2 against the running maximum, and K and V
+//                 accumulated in fp32 pairs (f32x2) with one rounding to the
+//                 storage type at the end.
 //
-// With w_eff = 1 (layers before l0) every row is a bit-exact copy.
+// Loaded vectors stay packed (16 bytes in four 32-bit registers) until they
+// are used, which keeps the kernel small enough for several CTAs per SM: the
+// loads of one warp are few, so the bandwidth comes from many warps in flight.
 #include <math.h>
 
 #include "common.cuh"
@@ -26,21 +31,56 @@
 namespace speechkv {
 namespace {
 
-constexpr int kPoolWarps = 8;
-constexpr int kPoolFrames = 4;  // frames of a window loaded at once
+constexpr int kPoolThreads = 256;
+constexpr int kPoolWarps = kPoolThreads / 32;
+constexpr int kPoolMinCtas = 2;   // CTAs per SM the register budget is set for
+constexpr int kPoolFrames = 4;    // frames of a window loaded at once
+constexpr int kCopyUnroll = 4;    // (K, V) vector pairs in flight per thread, copy phase
 
 template <typename T, int D>
 struct PoolCfg {
     static constexpr int kEpv = 16 / (int)sizeof(T);             // elements per 16-byte vector
     static constexpr int kVecPerHead = D * (int)sizeof(T) / 16;  // 8, 16 or 32
-    static constexpr int kHeadsPerChunk = 2048 / (D * (int)sizeof(T));
-    static constexpr int kVpl = kHeadsPerChunk * kVecPerHead / 32;  // vectors per lane
+    static constexpr int kHeadsPerWarp = 32 / kVecPerHead;       // heads of one pooled task
     static_assert(kVecPerHead <= 32 && 32 % kVecPerHead == 0, "head layout");
-    static_assert(kVpl >= 1 && kVpl * 32 * 16 == 2048, "chunk layout");
 };
 
+// 16 bytes of T, widened to fp32 pairs (element 2k, 2k + 1 in pair k).
+template <typename T>
+__device__ __forceinline__ void widen2(const uint4 &r, float2 (&f)[8 / sizeof(T)]) {
+    if constexpr (sizeof(T) == 4) {
+        f[0] = make_float2(__uint_as_float(r.x), __uint_as_float(r.y));
+        f[1] = make_float2(__uint_as_float(r.z), __uint_as_float(r.w));
+    } else {
+        f[0] = bf16x2_to_float2(r.x);
+        f[1] = bf16x2_to_float2(r.y);
+        f[2] = bf16x2_to_float2(r.z);
+        f[3] = bf16x2_to_float2(r.w);
+    }
+}
+
+// The same widening by byte permutes.  The accumulation pass uses this form
+// so that the compiler does not keep the logit pass's widened keys alive
+// (twice the registers of the packed words) to reuse them.
+template <typename T>
+__device__ __forceinline__ void widen2_prmt(const uint4 &r, float2 (&f)[8 / sizeof(T)]) {
+    if constexpr (sizeof(T) == 4) {
+        widen2<T>(r, f);
+    } else {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int k = 0; k < 4; k++) {
+            uint32_t lo, hi;
+            // bytes 4..7 come from the zero operand: lo = w << 16, hi = w & 0xffff0000
+            asm("prmt.b32 %0, %1, 0, 0x1054;" : "=r"(lo) : "r"(w[k]));
+            asm("prmt.b32 %0, %1, 0, 0x3254;" : "=r"(hi) : "r"(w[k]));
+            f[k] = make_float2(__uint_as_float(lo), __uint_as_float(hi));
+        }
+    }
+}
+
 template <typename T, int D>
-__global__ void __launch_bounds__(kPoolWarps * 32)
+__global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
     pool_kernel(const T *__restrict__ kf, const T *__restrict__ vf,
                 const int64_t *__restrict__ full_off, const int32_t *__restrict__ Pa,
                 const int32_t *__restrict__ Ta, const int32_t *__restrict__ Na,
@@ -48,7 +88,7 @@ __global__ void __launch_bounds__(kPoolWarps * 32)
                 const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
                 int64_t full_rows, int H_kv, int w, int *__restrict__ err) {
     using C = PoolCfg<T, D>;
-    constexpr int VPL = C::kVpl, EPV = C::kEpv, VH = C::kVecPerHead;
+    constexpr int EPV = C::kEpv, VH = C::kVecPerHead, HW = C::kHeadsPerWarp, NP = EPV / 2;
     const int b = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -69,122 +109,178 @@ __global__ void __launch_bounds__(kPoolWarps * 32)
     if (bad) return;
     const int64_t rows_out = L < cap ? L : cap;  // rows beyond the capacity are not written
 
-    const int nchunk = (H_kv + C::kHeadsPerChunk - 1) / C::kHeadsPerChunk;
-    const int64_t tasks = rows_out * nchunk;
-    const int64_t rowstride = (int64_t)H_kv * D;  // elements per prefill row
+    const int64_t VR = (int64_t)H_kv * VH;  // 16-byte vectors per prefill row
+    const uint4 *kb = reinterpret_cast<const uint4 *>(kf) + row0 * VR;
+    const uint4 *vb = reinterpret_cast<const uint4 *>(vf) + row0 * VR;
+    auto dst_off = [&](int64_t t, int64_t v) {  // element offset of (row t, vector v)
+        const int64_t h = v / VH;
+        return (base * H_kv + h * cap + t) * D + (v - h * VH) * EPV;
+    };
+
+    // ---- copy phase: copy row r is output row r for r < Pc, else the text
+    // row after the speech; with w = 1 every row is a copy row.
+    const int64_t Pc = w == 1 ? rows_out : (Pb < rows_out ? Pb : rows_out);
+    const int64_t after0 = Pb + n;  // first output row after the speech
+    const int64_t Ccopy = w == 1 ? rows_out : Pc + (rows_out > after0 ? rows_out - after0 : 0);
+    {
+        const int64_t g = (int64_t)blockIdx.x * kPoolThreads + threadIdx.x;
+        const int64_t Sg = (int64_t)gridDim.x * kPoolThreads;
+        int64_t r = g / VR, v = g - r * VR;
+        const int64_t dr = Sg / VR, dv = Sg - dr * VR;
+        while (r < Ccopy) {
+            uint4 kx[kCopyUnroll], vx[kCopyUnroll];
+            int64_t o[kCopyUnroll];  // destination element offset, -1 past the end
+#pragma unroll
+            for (int k = 0; k < kCopyUnroll; k++) {
+                o[k] = -1;
+                if (r < Ccopy) {
+                    const bool before = r < Pc;
+                    const int64_t src = before ? r : r - Pc + Pb + Tb;  // prefill row
+                    kx[k] = __ldcs(kb + src * VR + v);
+                    vx[k] = __ldcs(vb + src * VR + v);
+                    o[k] = dst_off(before ? r : r - Pc + after0, v);
+                }
+                r += dr;
+                v += dv;
+                if (v >= VR) {
+                    v -= VR;
+                    r++;
+                }
+            }
+#pragma unroll
+            for (int k = 0; k < kCopyUnroll; k++) {
+                if (o[k] < 0) break;  // the rows of later k are larger
+                *reinterpret_cast<uint4 *>(kc + o[k]) = kx[k];
+                *reinterpret_cast<uint4 *>(vc + o[k]) = vx[k];
+            }
+        }
+    }
+
+    // ---- pooled phase: windows i < npool (those that fit the capacity)
+    if (w == 1) return;
+    const int64_t room = rows_out - Pb;
+    const int64_t npool = room <= 0 ? 0 : (room < n ? room : n);
+    const int nchunk = (H_kv + HW - 1) / HW;
+    const int64_t tasks = npool * nchunk;
+    constexpr float kLog2e = 1.4426950408889634f;
     for (int64_t task = (int64_t)blockIdx.x * kPoolWarps + warp; task < tasks;
          task += (int64_t)gridDim.x * kPoolWarps) {
-        const int64_t t = task / nchunk;
-        const int h0 = (int)(task - t * nchunk) * C::kHeadsPerChunk;
-        const int hc = H_kv - h0 < C::kHeadsPerChunk ? H_kv - h0 : C::kHeadsPerChunk;
-        const int nv = hc * VH;  // vectors of this chunk
-        // the lane's vectors: v = lane + 32 i, of head h0 + v / VH
-        bool act[VPL];
-        int hv[VPL], cv[VPL];
-#pragma unroll
-        for (int i = 0; i < VPL; i++) {
-            const int v = lane + 32 * i;
-            act[i] = v < nv;
-            hv[i] = h0 + v / VH;
-            cv[i] = (v % VH) * EPV;
-        }
-        auto dst_of = [&](T *cache, int i) {
-            return cache + (base * H_kv + (int64_t)hv[i] * cap + t) * D + cv[i];
-        };
-        // prefill row 0 of request b, this lane's first vector of the chunk
-        const T *kb = kf + row0 * rowstride + (int64_t)h0 * D + lane * EPV;
-        const T *vb = vf + row0 * rowstride + (int64_t)h0 * D + lane * EPV;
-
-        if (t < Pb || t >= Pb + n || w == 1) {
-            // text row (or no pooling): bit-exact copy
-            const int64_t src = (t < Pb || w == 1) ? t : t - n + Tb;
-#pragma unroll
-            for (int i = 0; i < VPL; i++) {
-                if (!act[i]) continue;
-                copy_bytes<16>(dst_of(kc, i), kb + src * rowstride + 32 * i * EPV);
-                copy_bytes<16>(dst_of(vc, i), vb + src * rowstride + 32 * i * EPV);
-            }
-            continue;
-        }
-
-        // pooled speech row: frames [j0, j1) of the prefill rows
-        const int64_t j0 = Pb + (t - Pb) * w;
+        const int64_t i = task / nchunk;
+        const int64_t vi = (task - i * nchunk) * 32 + lane;  // this lane's vector of the row
+        const bool act = vi < VR;
+        const int64_t j0 = Pb + i * w;
         const int64_t j1 = (j0 + w < Pb + Tb) ? j0 + w : Pb + Tb;
-        float u[VPL][EPV];
+
+        // the lane's slice of the gate, scaled by log2(e): the softmax runs
+        // in base 2 (2^(log2(e) z) = e^z)
+        float2 u[NP];
+        if (act) {
+            const float4 *gp = reinterpret_cast<const float4 *>(gate + vi * EPV);
 #pragma unroll
-        for (int i = 0; i < VPL; i++)
+            for (int k = 0; k < NP; k += 2) {
+                const float4 g4 = __ldg(gp + k / 2);
+                u[k] = make_float2(g4.x * kLog2e, g4.y * kLog2e);
+                u[k + 1] = make_float2(g4.z * kLog2e, g4.w * kLog2e);
+            }
+        } else {
 #pragma unroll
-            for (int e = 0; e < EPV; e++)
-                u[i][e] = act[i] ? __ldg(gate + hv[i] * D + cv[i] + e) : 0.f;
-        float mx[VPL], sum[VPL], ak[VPL][EPV], av[VPL][EPV];
-#pragma unroll
-        for (int i = 0; i < VPL; i++) {
-            mx[i] = -INFINITY;
-            sum[i] = 0.f;
-#pragma unroll
-            for (int e = 0; e < EPV; e++) ak[i][e] = av[i][e] = 0.f;
+            for (int k = 0; k < NP; k++) u[k] = make_float2(0.f, 0.f);
         }
-        for (int64_t j = j0; j < j1; j += kPoolFrames) {
-            float kx[kPoolFrames][VPL][EPV], vx[kPoolFrames][VPL][EPV];
+        float m = -INFINITY, s = 0.f;
+        float2 ak[NP], av[NP];
 #pragma unroll
-            for (int f = 0; f < kPoolFrames; f++)
-#pragma unroll
-                for (int i = 0; i < VPL; i++) {
-                    if (j + f < j1 && act[i]) {
-                        load_vec<T, EPV>(kb + (j + f) * rowstride + 32 * i * EPV, kx[f][i]);
-                        load_vec<T, EPV>(vb + (j + f) * rowstride + 32 * i * EPV, vx[f][i]);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < EPV; e++) kx[f][i][e] = vx[f][i][e] = 0.f;
-                    }
-                }
+        for (int k = 0; k < NP; k++) ak[k] = av[k] = make_float2(0.f, 0.f);
+
+        const uint4 *kp = kb + j0 * VR + vi, *vp = vb + j0 * VR + vi;
+        for (int64_t j = j0; j < j1; j += kPoolFrames, kp += kPoolFrames * VR, vp += kPoolFrames * VR) {
+            const int nf = j1 - j < kPoolFrames ? (int)(j1 - j) : kPoolFrames;
+            uint4 kr[kPoolFrames], vr[kPoolFrames];
 #pragma unroll
             for (int f = 0; f < kPoolFrames; f++) {
-                if (j + f >= j1) break;
-#pragma unroll
-                for (int i = 0; i < VPL; i++) {
-                    // logit of this vector's head: reduce over its VH lanes
-                    float z = 0.f;
-#pragma unroll
-                    for (int e = 0; e < EPV; e++) z = fmaf(u[i][e], kx[f][i][e], z);
-#pragma unroll
-                    for (int o = 1; o < VH; o <<= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
-                    const float mnew = fmaxf(mx[i], z);
-                    const float corr = expf(mx[i] - mnew);  // 0 on the first frame
-                    const float p = expf(z - mnew);
-                    sum[i] = sum[i] * corr + p;
-#pragma unroll
-                    for (int e = 0; e < EPV; e++) {
-                        ak[i][e] = fmaf(p, kx[f][i][e], ak[i][e] * corr);
-                        av[i][e] = fmaf(p, vx[f][i][e], av[i][e] * corr);
-                    }
-                    mx[i] = mnew;
+                if (act && f < nf) {
+                    kr[f] = __ldcs(kp + f * VR);
+                    vr[f] = __ldcs(vp + f * VR);
+                } else {
+                    kr[f] = vr[f] = make_uint4(0u, 0u, 0u, 0u);
                 }
             }
-        }
+            // base-2 logits of the frames, reduced over the head's lanes
+            float z[kPoolFrames];
+            float mb = m;
 #pragma unroll
-        for (int i = 0; i < VPL; i++) {
-            if (!act[i]) continue;
-            const float inv = 1.f / sum[i];
+            for (int f = 0; f < kPoolFrames; f++) {
+                float2 x[NP];
+                widen2<T>(kr[f], x);
+                float2 a2 = fmul2(u[0], x[0]);
 #pragma unroll
-            for (int e = 0; e < EPV; e++) {
-                ak[i][e] *= inv;
-                av[i][e] *= inv;
+                for (int k = 1; k < NP; k++) a2 = ffma2(u[k], x[k], a2);
+                float acc = a2.x + a2.y;
+#pragma unroll
+                for (int o = 1; o < VH; o <<= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+                z[f] = acc;
+                if (f < nf) mb = fmaxf(mb, acc);
             }
-            store_vec<T, EPV>(dst_of(kc, i), ak[i]);
-            store_vec<T, EPV>(dst_of(vc, i), av[i]);
+            if (j != j0) {  // rescale what the earlier frames of the window left
+                const float corr = fast_exp2(m - mb);
+                const float2 c2 = make_float2(corr, corr);
+                s *= corr;
+#pragma unroll
+                for (int k = 0; k < NP; k++) {
+                    ak[k] = fmul2(ak[k], c2);
+                    av[k] = fmul2(av[k], c2);
+                }
+            }
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++) {
+                if (f >= nf) break;
+                const float p = fast_exp2(z[f] - mb);
+                const float2 p2 = make_float2(p, p);
+                s += p;
+                float2 xk[NP], xv[NP];
+                widen2_prmt<T>(kr[f], xk);
+                widen2_prmt<T>(vr[f], xv);
+#pragma unroll
+                for (int k = 0; k < NP; k++) {
+                    ak[k] = ffma2(p2, xk[k], ak[k]);
+                    av[k] = ffma2(p2, xv[k], av[k]);
+                }
+            }
+            m = mb;
+        }
+        if (act) {
+            const float inv = 1.f / s;
+            float ok[EPV], ov[EPV];
+#pragma unroll
+            for (int k = 0; k < NP; k++) {
+                ok[2 * k] = ak[k].x * inv;
+                ok[2 * k + 1] = ak[k].y * inv;
+                ov[2 * k] = av[k].x * inv;
+                ov[2 * k + 1] = av[k].y * inv;
+            }
+            const int64_t o = dst_off(Pb + i, vi);
+            store_vec<T, EPV>(kc + o, ok);
+            store_vec<T, EPV>(vc + o, ov);
         }
     }
 }
 
 template <typename T, int D>
 cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t stream) {
-    // about four CTAs per SM over the whole batch, at least one per request
-    int x = (4 * num_sms + a.B - 1) / a.B;
+    // enough CTAs over the whole batch to fill every SM once, at least one
+    // per request
+    static int per_sm = 0;
+    if (per_sm == 0) {
+        int occ = 0;
+        cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, pool_kernel<T, D>,
+                                                                      kPoolThreads, 0);
+        if (e != cudaSuccess) return e;
+        per_sm = occ > 0 ? occ : 1;
+    }
+    int64_t x = ((int64_t)per_sm * num_sms + a.B - 1) / a.B;
     if (x < 1) x = 1;
     if (x > 65535) x = 65535;
     const dim3 grid((unsigned)x, (unsigned)a.B);
-    pool_kernel<T, D><<<grid, kPoolWarps * 32, 0, stream>>>(
+    pool_kernel<T, D><<<grid, kPoolThreads, 0, stream>>>(
         static_cast<const T *>(a.k_full), static_cast<const T *>(a.v_full), a.full_off, a.P, a.T,
         a.N, a.gate, static_cast<T *>(a.k_cache), static_cast<T *>(a.v_cache), a.cache_off,
         a.len, a.full_rows, a.H_kv, a.w_eff, a.err);
