@@ -224,9 +224,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int64_t Cn = U < (int64_t)gridDim.x ? U : (int64_t)gridDim.x;
     const int64_t c = blockIdx.x;
     // Work that reads what the previous kernel may produce (k_new, v_new) or
-    // writes global memory waits for it.  The producer is the first warp to
-    // wait (after its first copies); the others do this part only once the
-    // first tile -- whose queries are copied after that wait -- has landed.
+    // writes global memory waits for it.  The producer waits after its first
+    // copies, the merge warp (idle until the first piece) at once, and the
+    // consumers only once the first tile -- whose queries are copied after
+    // that wait -- has landed.
     auto merge_warp_prior_part = [&]() {  // merge warp
         griddep_wait();
         // empty requests get a zero output (softmax over nothing)
@@ -381,15 +382,21 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         // ======== merge warp: combines the consumers' states of each piece ====
         // lane owns kCols consecutive output columns of every query head
         constexpr int kCols = D / 32;
-        constexpr int kBatch = 8;  // partials fetched per round of the final merge
-        int64_t k = 0;             // piece index within this CTA
+        // partials fetched per round of the final merge (every query head of
+        // a partial in the same round)
+        constexpr int kBatch = G >= 8 ? 1 : 8 / G;
+        // The merge warp idles until the first piece is deposited: it does
+        // its share of the work that waits for the previous kernel now, so
+        // that the done-counter round trip is not on the path of a CTA whose
+        // only piece ends with the kernel.
+        merge_warp_prior_part();
+        int64_t k = 0;  // piece index within this CTA
         for (int64_t u = u0; u < u1; k++) {
             const Piece p = piece_at(cum, B, H_kv, u, u1);
             const int x = (int)(k & 1);
             const uint32_t use = (uint32_t)((k >> 1) & 1);
             bool ok = !flags[0] && mbar_wait_bounded(&piece_bar[x], use, err);
             ok = __all_sync(0xffffffffu, ok) && !__shfl_sync(0xffffffffu, flags[0], 0);
-            if (k == 0) merge_warp_prior_part();
             const float *mo = mrg + x * C::kMergeFloats;  // [W][G][D]
             const float *mm = mo + W * G * D;              // [W][G]
             const float *ml = mm + W * G;                  // [W][G]
@@ -443,52 +450,60 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 last = __shfl_sync(0xffffffffu, last, 0);
                 __syncwarp();  // lane 0's acquire orders the other lanes' reads too
                 if (last) {
-#pragma unroll 1
+                    // online log-sum-exp over the pieces, per query head g;
+                    // kBatch partials (all heads) in flight per round
+                    float M[G], Ls[G], acc[G][kCols];
+#pragma unroll
                     for (int g = 0; g < G; g++) {
-                        // online log-sum-exp over the pieces, kBatch loads in flight
-                        float M = -INFINITY, Ls = 0.f, acc[kCols];
+                        M[g] = -INFINITY;
+                        Ls[g] = 0.f;
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[i] = 0.f;
+                        for (int i = 0; i < kCols; i++) acc[g][i] = 0.f;
+                    }
 #pragma unroll 1
-                        for (int64_t c0 = cfirst; c0 <= clast; c0 += kBatch) {
-                            float bm[kBatch], bl[kBatch], bo[kBatch][kCols];
+                    for (int64_t c0 = cfirst; c0 <= clast; c0 += kBatch) {
+                        float bm[kBatch][G], bl[kBatch][G], bo[kBatch][G][kCols];
 #pragma unroll
-                            for (int j = 0; j < kBatch; j++) {
-                                bm[j] = -INFINITY;
-                                bl[j] = 0.f;
+                        for (int j = 0; j < kBatch; j++) {
+                            const bool have = c0 + j <= clast;
+                            const float *sp = partials + (c0 + j + seg) * slot_floats;
 #pragma unroll
-                                for (int i = 0; i < kCols; i++) bo[j][i] = 0.f;
-                                if (c0 + j <= clast) {
-                                    const float *sp = partials + (c0 + j + seg) * slot_floats;
-                                    bm[j] = __ldcg(sp + G * D + g);
-                                    bl[j] = __ldcg(sp + G * D + G + g);
+                            for (int g = 0; g < G; g++) {
+                                bm[j][g] = have ? __ldcg(sp + G * D + g) : -INFINITY;
+                                bl[j][g] = have ? __ldcg(sp + G * D + G + g) : 0.f;
 #pragma unroll
-                                    for (int i = 0; i < kCols; i++)
-                                        bo[j][i] = __ldcg(sp + g * D + lane * kCols + i);
-                                }
+                                for (int i = 0; i < kCols; i++)
+                                    bo[j][g][i] = have ? __ldcg(sp + g * D + lane * kCols + i) : 0.f;
                             }
-                            float Mn = M;
-#pragma unroll
-                            for (int j = 0; j < kBatch; j++) Mn = fmaxf(Mn, bm[j]);
-                            const float r = fast_exp2(M - Mn);  // 0 while M = -inf
-                            Ls *= r;
-#pragma unroll
-                            for (int i = 0; i < kCols; i++) acc[i] *= r;
-#pragma unroll
-                            for (int j = 0; j < kBatch; j++) {
-                                const float sc = fast_exp2(bm[j] - Mn);  // absent: 0
-                                Ls = fmaf(bl[j], sc, Ls);
-#pragma unroll
-                                for (int i = 0; i < kCols; i++) acc[i] = fmaf(bo[j][i], sc, acc[i]);
-                            }
-                            M = Mn;
                         }
-                        const float inv = 1.f / Ls;
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[i] *= inv;
+                        for (int g = 0; g < G; g++) {
+                            float Mn = M[g];
+#pragma unroll
+                            for (int j = 0; j < kBatch; j++) Mn = fmaxf(Mn, bm[j][g]);
+                            const float r = fast_exp2(M[g] - Mn);  // 0 while M = -inf
+                            Ls[g] *= r;
+#pragma unroll
+                            for (int i = 0; i < kCols; i++) acc[g][i] *= r;
+#pragma unroll
+                            for (int j = 0; j < kBatch; j++) {
+                                const float sc = fast_exp2(bm[j][g] - Mn);  // absent: 0
+                                Ls[g] = fmaf(bl[j][g], sc, Ls[g]);
+#pragma unroll
+                                for (int i = 0; i < kCols; i++)
+                                    acc[g][i] = fmaf(bo[j][g][i], sc, acc[g][i]);
+                            }
+                            M[g] = Mn;
+                        }
+                    }
+#pragma unroll
+                    for (int g = 0; g < G; g++) {
+                        const float inv = 1.f / Ls[g];
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) acc[g][i] *= inv;
                         store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
                                                 lane * kCols,
-                                            acc);
+                                            acc[g]);
                     }
                     if (lane == 0) counters[seg] = 0;
                 }
