@@ -396,7 +396,10 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
 def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_key: int,
                 layers=None):
     """Same decode steps through the C ABI with HOST buffers: every step copies
-    its q/k/v from pinned host memory and reads the outputs back."""
+    its q/k/v (all layers, one copy per tensor) from pinned host memory, runs
+    the layers' fused decode steps back to back (consecutive layers may
+    overlap, as in the device-resident passes) and reads the outputs of all
+    layers back in one copy."""
     import torch
     model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key, layers=layers)
     L, B, Hq, Hk, d = len(model.layers), wl.B, wl.H_q, wl.H_kv, wl.d
@@ -411,13 +414,16 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
     sk = model.sk
 
     def step(s):
+        d_q.copy_(h_q[s], non_blocking=True)
+        d_kn.copy_(h_kn[s], non_blocking=True)
+        d_vn.copy_(h_vn[s], non_blocking=True)
         for i, layer in enumerate(model.layers):
-            d_q[i].copy_(h_q[s, i], non_blocking=True)
-            d_kn[i].copy_(h_kn[s, i], non_blocking=True)
-            d_vn[i].copy_(h_vn[s, i], non_blocking=True)
+            # after the first layer the previous kernel is another layer's
+            # decode step, which writes none of this layer's cache or length
             sk.decode_step(d_q[i], d_kn[i], d_vn[i], model.k[i], model.v[i], model.off[i],
-                           model.len[i], model.out[i], model.ws, wl.w, layer, wl.l0)
-            h_out[s, i].copy_(model.out[i], non_blocking=True)
+                           model.len[i], model.out[i], model.ws, wl.w, layer, wl.l0,
+                           flags=sk.OVERLAP_PRIOR if i > 0 else 0)
+        h_out[s].copy_(model.out, non_blocking=True)
 
     for s in range(warmup):
         step(s)
