@@ -68,6 +68,13 @@ def _load():
         lib.oracle_decode_attn_request.argtypes = [
             _D, _D, _D, ctypes.c_int64, ctypes.c_int32, ctypes.c_int32,
             ctypes.c_int32, ctypes.c_double, ctypes.c_int32, _D, _D]
+        lib.oracle_prefill_position.restype = ctypes.c_int64
+        lib.oracle_prefill_position.argtypes = [ctypes.c_int32] * 4 + [ctypes.c_int64]
+        lib.oracle_prefill_attn_request.restype = ctypes.c_int32
+        lib.oracle_prefill_attn_request.argtypes = [
+            _D, _D, _D, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, ctypes.c_int32,
+            ctypes.c_double, ctypes.c_int32, _D]
         _lib = lib
         return lib
 
@@ -148,3 +155,31 @@ def decode_attn_request(q, K, V, scale: float = 0.0,
     if rc != 0:
         raise ValueError("oracle_decode_attn_request: bad arguments")
     return (out, probs) if want_probs else out
+
+
+def prefill_position(P: int, T: int, N: int, w_eff: int, t: int) -> int:
+    """Compressed row holding prompt position t (the query's place in the
+    compressed sequence for the prefill mask)."""
+    r = _load().oracle_prefill_position(P, T, N, w_eff, t)
+    if r < 0:
+        raise ValueError("oracle_prefill_position: bad arguments")
+    return r
+
+
+def prefill_attn_request(Q, K, V, P: int, T: int, N: int, w_eff: int,
+                         scale: float = 0.0, storage: int = STORE_EXACT):
+    """Eq. (attn) at prefill with the adjusted causal mask, one request.
+    Q: [P + T + N, H_q, d]; K, V: compressed [c, H_kv, d].  Returns
+    out [P + T + N, H_q, d]."""
+    Q, K, V = _f64(Q), _f64(K), _f64(V)
+    S, H_q, d = Q.shape
+    c, H_kv, d2 = K.shape
+    assert S == P + T + N and d2 == d and V.shape == K.shape
+    assert c == compressed_len(P, T, N, 0, w_eff, 0, 0)
+    out = np.zeros((S, H_q, d))
+    rc = _load().oracle_prefill_attn_request(
+        _ptr(Q), _ptr(K), _ptr(V), P, T, N, w_eff, H_q, H_kv, d, float(scale),
+        storage, _ptr(out))
+    if rc != 0:
+        raise ValueError("oracle_prefill_attn_request: bad arguments")
+    return out

@@ -18,6 +18,14 @@
  *   Decode attention: at every layer the full-resolution query attends over
  *   the (compressed) cache, softmax(q K^T / sqrt(d_h)) V, grouped-query style.
  *
+ *   Prefill attention (Sec. III-B, Eq. (attn) with the adjusted causal mask):
+ *   every full-resolution prompt query attends over the compressed rows that
+ *   precede it.  Reading of "causality over the compressed sequence": a
+ *   query at prompt position t is placed at the compressed position pi(t)
+ *   of the row that holds it (t for the text prefix, P + floor((t - P) / w)
+ *   for a speech frame -- its own window --, t - T + n for the text after
+ *   the speech) and sees compressed rows 0 .. pi(t).
+ *
  * Everything is plain loops in fp64 written straight from those
  * definitions.  No blocking, no fusion, no online softmax.  Readings of
  * points the paper leaves open (see the design notes of the repository):
@@ -260,6 +268,83 @@ int32_t oracle_decode_attn_request(const double *q, const double *K,
             for (int64_t j = 0; j < n; j++)
                 acc += p[j] * V[j * row + (int64_t)h * d + c];
             out[(int64_t)hq * d + c] = store(acc, storage);
+        }
+    }
+    free(p);
+    return 0;
+}
+
+/* Compressed position of prompt position t (0 <= t < P + T + N) at window
+ * w_eff: the row of the compressed cache that holds position t.  -1 on bad
+ * arguments. */
+int64_t oracle_prefill_position(int32_t P, int32_t T, int32_t N, int32_t w_eff,
+                                int64_t t)
+{
+    if (P < 0 || T < 0 || N < 0 || w_eff < 1 || t < 0 ||
+        t >= (int64_t)P + T + N)
+        return -1;
+    int64_t n = 0;
+    while (n * w_eff < T)
+        n++;
+    if (t < P)
+        return t;
+    if (t < (int64_t)P + T)
+        return P + (t - P) / w_eff;
+    return t - T + n;
+}
+
+/* Eq. (attn) at prefill for one request: Q [S][H_q][d] (S = P + T + N
+ * prompt positions), compressed K, V [c][H_kv][d] (c = P + n + N rows, as
+ * the pooling writes them), out [S][H_q][d].  Query t, head hq attends over
+ * rows 0 .. pi(t) of KV head hq / (H_q / H_kv) with weights
+ * softmax(q . k / sqrt(d)) (scale <= 0 means 1 / sqrt(d)). */
+int32_t oracle_prefill_attn_request(const double *Q, const double *K,
+                                    const double *V, int32_t P, int32_t T,
+                                    int32_t N, int32_t w_eff, int32_t H_q,
+                                    int32_t H_kv, int32_t d, double scale,
+                                    int32_t storage, double *out)
+{
+    if (H_q < 1 || H_kv < 1 || d < 1 || H_q % H_kv != 0 || P < 0 || T < 0 ||
+        N < 0 || w_eff < 1)
+        return -1;
+    if (!(scale > 0.0))
+        scale = 1.0 / sqrt((double)d);
+    const int64_t S = (int64_t)P + T + N;
+    int64_t n = 0;
+    while (n * w_eff < T)
+        n++;
+    const int64_t c = P + n + N;
+    const int32_t group = H_q / H_kv;
+    const int64_t qrow = (int64_t)H_q * d, krow = (int64_t)H_kv * d;
+    double *p = (double *)malloc(sizeof(double) * (size_t)(c > 0 ? c : 1));
+    if (!p)
+        return -1;
+    for (int64_t t = 0; t < S; t++) {
+        const int64_t last = oracle_prefill_position(P, T, N, w_eff, t);
+        for (int32_t hq = 0; hq < H_q; hq++) {
+            const int32_t h = hq / group;
+            const double *q = Q + t * qrow + (int64_t)hq * d;
+            for (int64_t e = 0; e <= last; e++) {
+                double s = 0.0;
+                for (int32_t k = 0; k < d; k++)
+                    s += q[k] * K[e * krow + (int64_t)h * d + k];
+                p[e] = s * scale;
+            }
+            double m = p[0];
+            for (int64_t e = 1; e <= last; e++)
+                if (p[e] > m)
+                    m = p[e];
+            double sum = 0.0;
+            for (int64_t e = 0; e <= last; e++) {
+                p[e] = exp(p[e] - m);
+                sum += p[e];
+            }
+            for (int32_t k = 0; k < d; k++) {
+                double acc = 0.0;
+                for (int64_t e = 0; e <= last; e++)
+                    acc += p[e] * V[e * krow + (int64_t)h * d + k];
+                out[t * qrow + (int64_t)hq * d + k] = store(acc / sum, storage);
+            }
         }
     }
     free(p);

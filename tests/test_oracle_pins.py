@@ -366,3 +366,116 @@ def test_w1_pipeline_is_uncompressed_attention(oracle):
         Kfull = np.concatenate([Kfull, kn[None]]); Vfull = np.concatenate([Vfull, vn[None]])
         np.testing.assert_allclose(oracle.decode_attn_request(q, Kc[:n], Vc[:n]),
                                    _sdpa_gqa(q, Kfull, Vfull), rtol=0, atol=1e-12)
+
+
+# --------------------------------------------------------------------------
+# prefill attention (Eq. (attn) with the adjusted causal mask)
+# --------------------------------------------------------------------------
+def _first_source(P, T, N, w):
+    """Prompt position of the first frame behind each compressed row: the
+    text prefix maps to itself, pooled window i starts at frame P + i*w, the
+    text after the speech sits T - n positions further on.  Written from the
+    row order of the compressed cache, not from the oracle."""
+    n = -(-T // w)
+    return [e for e in range(P)] + [P + i * w for i in range(n)] + \
+        [P + T + j for j in range(N)]
+
+
+def _visible(P, T, N, w):
+    """mask[t][e]: compressed row e precedes prompt position t (its first
+    source frame is not after t)."""
+    src = np.array(_first_source(P, T, N, w))
+    t = np.arange(P + T + N)
+    return src[None, :] <= t[:, None]
+
+
+@pytest.mark.parametrize("P,T,N,w", [(0, 375, 32, 4), (16, 64, 0, 4), (3, 10, 5, 3),
+                                     (2, 7, 3, 8), (0, 1, 1, 4), (5, 0, 4, 4), (4, 9, 2, 1)])
+def test_prefill_position_is_last_visible_row(oracle, P, T, N, w):
+    mask = _visible(P, T, N, w)
+    for t in range(P + T + N):
+        vis = np.nonzero(mask[t])[0]
+        # the visible rows are a prefix, and pi(t) is its last row
+        assert list(vis) == list(range(len(vis)))
+        assert oracle.prefill_position(P, T, N, w, t) == vis[-1]
+    assert oracle.prefill_position(P, T, N, w, P + T + N - 1) == mask.shape[1] - 1
+
+
+def _sdpa_causal(Q, K, V, mask=None):
+    """torch scaled_dot_product_attention in fp64, GQA by repeating KV heads."""
+    G = Q.shape[1] // K.shape[1]
+    qt = torch.from_numpy(Q).permute(1, 0, 2)
+    kt = torch.from_numpy(K).permute(1, 0, 2).repeat_interleave(G, 0)
+    vt = torch.from_numpy(V).permute(1, 0, 2).repeat_interleave(G, 0)
+    if mask is None:
+        o = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True)
+    else:
+        o = torch.nn.functional.scaled_dot_product_attention(
+            qt, kt, vt, attn_mask=torch.from_numpy(mask))
+    return o.permute(1, 0, 2).numpy()
+
+
+@pytest.mark.parametrize("P,T,N,H_q,H_kv,d", [(4, 30, 6, 4, 2, 16), (0, 50, 0, 2, 2, 8),
+                                              (7, 0, 3, 6, 3, 32)])
+def test_prefill_w1_is_causal_attention(oracle, P, T, N, H_q, H_kv, d):
+    """Without pooling the prefill is plain causal attention (the library's)."""
+    S = P + T + N
+    Q, K, V = _rand(90, S, H_q, d), _rand(91, S, H_kv, d), _rand(92, S, H_kv, d)
+    np.testing.assert_allclose(oracle.prefill_attn_request(Q, K, V, P, T, N, 1),
+                               _sdpa_causal(Q, K, V), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("P,T,N,w", [(0, 37, 8, 4), (5, 20, 3, 3), (2, 7, 0, 8)])
+def test_prefill_matches_masked_sdpa(oracle, P, T, N, w):
+    """Pooled layer: the library's attention with the mask of the window
+    sources gives the same rows."""
+    H_q, H_kv, d = 4, 2, 16
+    c = len(_first_source(P, T, N, w))
+    Q, K, V = _rand(93, P + T + N, H_q, d), _rand(94, c, H_kv, d), _rand(95, c, H_kv, d)
+    np.testing.assert_allclose(oracle.prefill_attn_request(Q, K, V, P, T, N, w),
+                               _sdpa_causal(Q, K, V, _visible(P, T, N, w)), rtol=0, atol=1e-12)
+
+
+def test_prefill_last_row_is_decode_attention(oracle):
+    """The last prompt position sees the whole compressed cache: its row is
+    the decode attention of that query."""
+    P, T, N, w, H_q, H_kv, d = 3, 41, 5, 4, 8, 4, 32
+    c = len(_first_source(P, T, N, w))
+    Q, K, V = _rand(96, P + T + N, H_q, d), _rand(97, c, H_kv, d), _rand(98, c, H_kv, d)
+    out = oracle.prefill_attn_request(Q, K, V, P, T, N, w)
+    np.testing.assert_allclose(out[-1], oracle.decode_attn_request(Q[-1], K, V),
+                               rtol=0, atol=1e-12)
+
+
+def test_prefill_equal_keys_average_visible_values(oracle):
+    """All keys of a head equal: the softmax is uniform, so each query gets
+    the running mean of the values it may see."""
+    P, T, N, w, H_q, H_kv, d = 2, 13, 3, 4, 4, 2, 8
+    mask = _visible(P, T, N, w)
+    c = mask.shape[1]
+    Q, V = _rand(99, P + T + N, H_q, d), _rand(100, c, H_kv, d)
+    K = np.repeat(_rand(101, 1, H_kv, d), c, axis=0)
+    out = oracle.prefill_attn_request(Q, K, V, P, T, N, w)
+    for t in range(P + T + N):
+        for hq in range(H_q):
+            ref = V[mask[t], hq // 2].mean(axis=0)
+            np.testing.assert_allclose(out[t, hq], ref, rtol=0, atol=1e-12)
+
+
+def test_prefill_brute_force_tiny_case(oracle):
+    """Explicit loops from the definitions: mask from the window sources,
+    exp without max subtraction, scale 1/sqrt(d)."""
+    P, T, N, w, H_q, H_kv, d = 2, 7, 3, 3, 4, 2, 8
+    mask = _visible(P, T, N, w)
+    c = mask.shape[1]
+    Q, K, V = _rand(102, P + T + N, H_q, d), _rand(103, c, H_kv, d), _rand(104, c, H_kv, d)
+    out = oracle.prefill_attn_request(Q, K, V, P, T, N, w)
+    for t in range(P + T + N):
+        for hq in range(H_q):
+            h = hq // (H_q // H_kv)
+            e = [math.exp(sum(Q[t, hq, k] * K[j, h, k] for k in range(d)) / math.sqrt(d))
+                 if mask[t, j] else 0.0 for j in range(c)]
+            tot = sum(e)
+            for k in range(d):
+                ref = sum(e[j] / tot * V[j, h, k] for j in range(c))
+                assert abs(out[t, hq, k] - ref) < 1e-12
