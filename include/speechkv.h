@@ -138,6 +138,55 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full,
                               speechkv_dtype dtype, cudaStream_t stream);
 
 /*
+ * speechkv_prefill_attn -- Eq. (attn) at prefill (Sec. III-B): every
+ * full-resolution prompt query attends over the compressed cache rows that
+ * precede it.
+ *
+ * The paper adjusts the causal mask so that a query sees only the positions
+ * before it, with causality taken over the compressed sequence.  Here a
+ * query at prompt position t (0 <= t < S_b = P + T + N) sits at compressed
+ * position
+ *     pi(t) = t                      (t < P, text before the speech)
+ *           = P + (t - P) / w_eff    (speech frame: the row of its window)
+ *           = t - T + n              (text after the speech)
+ * and attends, with weights softmax(q . k / sqrt(d)), over rows 0 .. pi(t)
+ * of its KV head (hq / (H_q / H_kv)).  With w_eff = 1 (layer < l0) this is
+ * ordinary causal attention.  The cache is read as speechkv_pool leaves it:
+ * rows 0 .. P + n + N - 1 of every (request, KV head).
+ *
+ * q           dev bf16 [q_rows][H_q][d], token-major prompt queries (after
+ *             any rotary embedding); request b's positions 0 .. S_b - 1 are
+ *             rows q_off[b] .. q_off[b+1] - 1.
+ * q_off       dev int64 [B+1], q_off[b+1] - q_off[b] must equal P+T+N.
+ * q_rows      host: rows of q and out.
+ * P, T, N     dev int32 [B], as for speechkv_pool.
+ * k_cache, v_cache, cache_off: this layer's cache (layout above).
+ * cache_rows  host: the cache buffers hold cache_rows * H_kv * d elements
+ *             (cache_off[B] <= cache_rows); reads never go past them.
+ * out         dev bf16 [q_rows][H_q][d]: row q_off[b] + t of head hq is
+ *             written for every t < S_b (other rows are left as they are).
+ * scale       0 for 1/sqrt(d), else the logit scale.
+ * w, layer, l0  w_eff = (layer >= l0 ? w : 1).
+ * Supported: SPEECHKV_BF16, d = 128, B <= SPEECHKV_MAX_BATCH, H_q <= 256,
+ * q_rows and cache_rows * H_kv below 2^31 (SPEECHKV_ERR_UNSUPPORTED
+ * otherwise).  On the device a request whose query rows do not match P+T+N
+ * (or lie outside q_rows / cache_rows) sets SPEECHKV_ERR_INVALID_ARG, one
+ * whose compressed rows exceed its capacity SPEECHKV_ERR_CAPACITY; such
+ * requests are skipped.
+ */
+speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off,
+                                      int64_t q_rows, const int32_t *P,
+                                      const int32_t *T, const int32_t *N,
+                                      const void *k_cache, const void *v_cache,
+                                      const int64_t *cache_off,
+                                      int64_t cache_rows, void *out,
+                                      float scale, int32_t B, int32_t H_q,
+                                      int32_t H_kv, int32_t d, int32_t w,
+                                      int32_t layer, int32_t l0,
+                                      speechkv_dtype dtype,
+                                      cudaStream_t stream);
+
+/*
  * speechkv_append -- one decode step's cache update (Sec. III-C: decoding
  * appends each new token to the cache uncompressed).
  *

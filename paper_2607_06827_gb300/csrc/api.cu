@@ -1,6 +1,6 @@
 // C ABI of libspeechkv: argument checks, per-device state and dispatch to the
-// kernels (pool.cu, append.cu, decode_attn.cu).  Declarations and the full
-// contract of every entry point are in include/speechkv.h.
+// kernels (pool.cu, append.cu, decode_attn.cu, prefill_attn.cu).  Declarations
+// and the full contract of every entry point are in include/speechkv.h.
 #include <math.h>
 #include <stdint.h>
 
@@ -235,6 +235,55 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full, const int6
     a.err = s->err;
     return speechkv::launch_pool(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
                                                                        : SPEECHKV_ERR_CUDA;
+}
+
+speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64_t q_rows,
+                                      const int32_t *P, const int32_t *T, const int32_t *N,
+                                      const void *k_cache, const void *v_cache,
+                                      const int64_t *cache_off, int64_t cache_rows, void *out,
+                                      float scale, int32_t B, int32_t H_q, int32_t H_kv,
+                                      int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                      speechkv_dtype dtype, cudaStream_t stream) {
+    if (B < 0 || B > SPEECHKV_MAX_BATCH || q_rows < 0 || cache_rows < 0 || H_q < 1 ||
+        H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype) ||
+        isnan(scale) || isinf(scale) || scale < 0.f)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!speechkv::prefill_supported(dtype, d)) return SPEECHKV_ERR_UNSUPPORTED;
+    // tensor-copy coordinates are 32-bit
+    if (q_rows >= (1ll << 31) || cache_rows * (int64_t)H_kv >= (1ll << 31) || H_q > 256)
+        return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0 || q_rows == 0) return SPEECHKV_OK;
+    if (!q || !q_off || !P || !T || !N || !k_cache || !v_cache || !cache_off || !out ||
+        cache_rows == 0)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
+        !aligned(q_off, 8) || !aligned(cache_off, 8) || !aligned(P, 4) || !aligned(T, 4) ||
+        !aligned(N, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::PrefillArgs a;
+    a.q = q;
+    a.q_off = q_off;
+    a.q_rows = q_rows;
+    a.P = P;
+    a.T = T;
+    a.N = N;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.cache_rows = cache_rows;
+    a.out = out;
+    a.scale = scale > 0.f ? scale : 1.f / sqrtf((float)d);
+    a.B = B;
+    a.H_q = H_q;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.w_eff = layer >= l0 ? w : 1;
+    a.err = s->err;
+    return speechkv::launch_prefill(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                          : SPEECHKV_ERR_CUDA;
 }
 
 speechkv_status speechkv_append(const void *k_new, const void *v_new, void *k_cache,

@@ -62,4 +62,21 @@ int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B);
 int decode_slot_floats(int d, int group);
 cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream);
 
+struct PrefillArgs {
+    const void *q;  // [q_rows][H_q][d]
+    const int64_t *q_off;
+    int64_t q_rows;
+    const int32_t *P, *T, *N;
+    const void *k_cache, *v_cache;
+    const int64_t *cache_off;
+    int64_t cache_rows;  // rows per KV head block extent: buffers hold cache_rows * H_kv * d
+    void *out;           // [q_rows][H_q][d]
+    float scale;         // > 0
+    int32_t B, H_q, H_kv, d, w_eff;
+    int *err;
+};
+// Whether (dtype, d) has a compiled prefill kernel.
+bool prefill_supported(speechkv_dtype dtype, int d);
+cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t stream);
+
 }  // namespace speechkv

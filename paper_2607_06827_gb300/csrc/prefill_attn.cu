@@ -1,0 +1,598 @@
+// speechkv_prefill_attn: Eq. (attn) at prefill (Sec. III-B) -- every
+// full-resolution prompt query attends over the compressed cache rows that
+// precede it.  A query at prompt position t sits at compressed position
+//   pi(t) = t                     text before the speech   (t < P)
+//         = P + (t - P) / w_eff   speech frame (its own window)
+//         = t - T + n             text after the speech
+// and sees rows 0 .. pi(t) (causality over the compressed sequence).
+//
+// Blackwell tensor-core flash attention, bf16 in, fp32 accumulate, d = 128:
+//   * persistent: one CTA per SM walks work items (request, query head,
+//     128-row query tile), heaviest tiles (latest prompt positions) first;
+//   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the query tile
+//     and of 128-row key and value tiles (two stages) from the cache;
+//   * warp 1 lane 0: tcgen05.mma issue -- S = Q K^T into a 128-column TMEM
+//     buffer, O += P V into another (V as the MN-major operand);
+//   * warps 2-5: softmax, one query row per thread (= TMEM lane): two passes
+//     over S in TMEM (row maximum, then base-2 exponentials with
+//     log2(e)/sqrt(d) folded in), P written as bf16 into shared memory in
+//     the MMA's swizzled K-major layout, O rescaled in TMEM when a warp's
+//     running maximum moved, and the epilogue O / l to global memory.
+// Cache rows past a request's compressed length are zeroed in the value
+// stage (their contents are unspecified and the MMA would multiply them by
+// zero weights: 0 x NaN is NaN).  Every wait is bounded; on a timeout the CTA
+// stops, lets its copies and MMAs finish and reports SPEECHKV_ERR_TIMEOUT.
+#include <cuda.h>
+#include <math.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace speechkv {
+namespace {
+
+constexpr int kBM = 128;  // query rows per tile = TMEM lanes
+constexpr int kBN = 128;  // keys per tile
+constexpr int kD = 128;   // head dimension
+constexpr int kThreads = 192;
+constexpr int kTileBytes = kBM * kD * 2;  // one bf16 tile of 128 rows x 128
+constexpr int kHalf = kTileBytes / 2;     // its 64-column block (128-byte rows)
+constexpr int kStages = 2;                // key/value ring
+constexpr uint32_t kTmemCols = 256;       // S: columns 0..127, O: 128..255
+
+// shared memory (offsets from a 1024-byte aligned base)
+constexpr int kOffQ = 0;
+constexpr int kOffK = kOffQ + kTileBytes;
+constexpr int kOffV = kOffK + kStages * kTileBytes;
+constexpr int kOffP = kOffV + kStages * kTileBytes;
+constexpr int kOffBar = kOffP + kTileBytes;
+enum Bar { kQFull, kQEmpty, kKFull, kVFull = kKFull + kStages, kKvEmpty = kVFull + kStages,
+           kSFull = kKvEmpty + kStages, kSFree, kPFull, kOFull, kDrain, kNumBars };
+constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem address, abort flag, largest tile count
+constexpr int kOffTab = kOffMisc + 16;
+
+struct Req {         // per-request table in shared memory
+    int64_t q0;      // first query row
+    int64_t kv0;     // cache_off[b]
+    int64_t cap;     // capacity (rows)
+    int32_t P, T, N, n, S, tiles;
+};
+static_assert(sizeof(Req) == 48, "table entry");
+
+size_t smem_bytes(int B) { return (size_t)kOffTab + (size_t)B * sizeof(Req) + 1024; }
+
+__device__ __forceinline__ int64_t pi_of(const Req &q, int64_t t, int w) {
+    if (t < q.P) return t;
+    if (t < (int64_t)q.P + q.T) return q.P + (t - q.P) / w;
+    return t - q.T + q.n;
+}
+
+// ---------------------------------------------------------------- tcgen05 --
+// Shared-memory matrix descriptor, 128-byte swizzle: start address, leading
+// and stride byte offsets (16-byte units), descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((addr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
+}
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, A
+// K-major, B K-major or MN-major, M = 128, N = 128.
+__device__ __forceinline__ uint32_t instr_desc(bool b_mn_major) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+           ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+}
+__device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
+                                     uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(id), "r"(accumulate));
+}
+// Arrive on `bar` once every tcgen05 operation issued so far by this thread
+// has completed.
+__device__ __forceinline__ void umma_commit(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+            taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+// TMA tensor copies global -> shared (completion as transaction bytes on bar)
+__device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x, int y,
+                                       uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, "
+        "{%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<unsigned long long>(map)), "r"(smem_addr(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+__device__ __forceinline__ void tma_3d(void *dst, const CUtensorMap *map, int x, int y, int z,
+                                       uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, "
+        "{%3, %4, %5}], [%2];" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<unsigned long long>(map)), "r"(smem_addr(bar)), "r"(x), "r"(y),
+        "r"(z)
+        : "memory");
+}
+
+// Bounded wait that also gives up once another role has aborted.
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatile int *abort,
+                                         int *err) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_timer_ns();
+    for (;;) {
+        for (int i = 0; i < 64; i++)
+            if (mbar_try_wait(bar, parity)) return true;
+        if (*abort) return false;
+        if (global_timer_ns() - t0 > kWaitLimitNs) {
+            report_error(err, SPEECHKV_ERR_TIMEOUT);
+            *abort = 1;
+            return false;
+        }
+    }
+}
+
+// Work item k of the CTA-independent order: query tile i (from the last
+// tile of the longest request down), then request, then query head.
+struct Item {
+    int b, hq, i;
+    bool valid;
+};
+__device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int B, int H_q,
+                                        const Req *tab) {
+    Item it;
+    const int64_t per = (int64_t)B * H_q;
+    it.i = tiles_max - 1 - (int)(k / per);
+    const int rem = (int)(k % per);
+    it.b = rem / H_q;
+    it.hq = rem - it.b * H_q;
+    it.valid = it.i < tab[it.b].tiles;
+    return it;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
+                        const __grid_constant__ CUtensorMap tm_k,
+                        const __grid_constant__ CUtensorMap tm_v,
+                        const int64_t *__restrict__ q_off, const int32_t *__restrict__ Pa,
+                        const int32_t *__restrict__ Ta, const int32_t *__restrict__ Na,
+                        const int64_t *__restrict__ cache_off, __nv_bfloat16 *__restrict__ out,
+                        int64_t q_rows, int64_t cache_rows, float sl2, int B, int H_q,
+                        int H_kv, int w, int *__restrict__ err) {
+    extern __shared__ unsigned char smem_raw[];
+    unsigned char *sm = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + kOffBar);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
+    volatile int *abort = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
+    int *tiles_max_s = reinterpret_cast<int *>(sm + kOffMisc + 8);
+    Req *tab = reinterpret_cast<Req *>(sm + kOffTab);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int G = H_q / H_kv;
+
+    // ---- prologue: barriers, TMEM, per-request table
+    if (tid == 0) {
+        mbar_init(&bar[kQFull], 1);
+        mbar_init(&bar[kQEmpty], 1);
+        for (int s = 0; s < kStages; s++) {
+            mbar_init(&bar[kKFull + s], 1);
+            mbar_init(&bar[kVFull + s], 1);
+            mbar_init(&bar[kKvEmpty + s], 1);
+        }
+        mbar_init(&bar[kSFull], 1);
+        mbar_init(&bar[kSFree], kBM);
+        mbar_init(&bar[kPFull], kBM);
+        mbar_init(&bar[kOFull], 1);
+        mbar_init(&bar[kDrain], 1);
+        fence_mbar_init();
+        *abort = 0;
+    }
+    if (warp == 1) {
+        asm volatile(
+            "tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                smem_addr(tmem_slot)),
+            "r"(kTmemCols)
+            : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    for (int b = tid; b < B; b += kThreads) {
+        Req q;
+        q.q0 = q_off[b];
+        const int64_t q1 = q_off[b + 1];
+        q.kv0 = cache_off[b];
+        const int64_t kv1 = cache_off[b + 1];
+        q.cap = kv1 - q.kv0;
+        q.P = Pa[b];
+        q.T = Ta[b];
+        q.N = Na[b];
+        q.n = q.T >= 0 ? (int32_t)(((int64_t)q.T + w - 1) / w) : 0;
+        const int64_t S = (int64_t)q.P + q.T + q.N;
+        const int64_t c = (int64_t)q.P + q.n + q.N;
+        q.S = (int32_t)S;
+        bool ok = q.P >= 0 && q.T >= 0 && q.N >= 0 && q.q0 >= 0 && q1 - q.q0 == S &&
+                  q1 <= q_rows && q.kv0 >= 0 && kv1 <= cache_rows && S < (1ll << 31);
+        if (!ok) {
+            if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
+        } else if (c > q.cap) {
+            if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_CAPACITY);
+            ok = false;
+        }
+        q.tiles = ok ? (int32_t)((S + kBM - 1) / kBM) : 0;
+        tab[b] = q;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        int mx = 0;
+        for (int b = lane; b < B; b += 32) mx = max(mx, tab[b].tiles);
+        for (int o = 16; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        if (lane == 0) *tiles_max_s = mx;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int tiles_max = *tiles_max_s;
+    const int64_t total = (int64_t)tiles_max * B * H_q;
+
+    unsigned char *sQ = sm + kOffQ, *sK = sm + kOffK, *sV = sm + kOffV, *sP = sm + kOffP;
+
+    if (warp == 0) {
+        // ===================== TMA producer =====================
+        if (lane == 0) {
+            int64_t it = 0, g = 0;
+            for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
+                const Item item = item_at(k, tiles_max, B, H_q, tab);
+                if (!item.valid) continue;
+                const Req &q = tab[item.b];
+                const int64_t t0 = (int64_t)item.i * kBM;
+                const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
+                const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
+                const int64_t kvrow = q.kv0 * H_kv + (int64_t)(item.hq / G) * q.cap;
+                if (it > 0 && !wait_bar(&bar[kQEmpty], (uint32_t)((it - 1) & 1), abort, err)) break;
+                mbar_arrive_expect_tx(&bar[kQFull], kTileBytes);
+                tma_3d(sQ, &tm_q, 0, item.hq, (int)(q.q0 + t0), &bar[kQFull]);
+                tma_3d(sQ + kHalf, &tm_q, 64, item.hq, (int)(q.q0 + t0), &bar[kQFull]);
+                ++it;
+                bool stop = false;
+                for (int j = 0; j < n_kt; j++, g++) {
+                    const int s = (int)(g & 1);
+                    if (g >= kStages &&
+                        !wait_bar(&bar[kKvEmpty + s], (uint32_t)(((g >> 1) - 1) & 1), abort, err)) {
+                        stop = true;
+                        break;
+                    }
+                    const int y = (int)(kvrow + (int64_t)j * kBN);
+                    mbar_arrive_expect_tx(&bar[kKFull + s], kTileBytes);
+                    tma_2d(sK + s * kTileBytes, &tm_k, 0, y, &bar[kKFull + s]);
+                    tma_2d(sK + s * kTileBytes + kHalf, &tm_k, 64, y, &bar[kKFull + s]);
+                    mbar_arrive_expect_tx(&bar[kVFull + s], kTileBytes);
+                    tma_2d(sV + s * kTileBytes, &tm_v, 0, y, &bar[kVFull + s]);
+                    tma_2d(sV + s * kTileBytes + kHalf, &tm_v, 64, y, &bar[kVFull + s]);
+                }
+                if (stop) break;
+            }
+            // let every copy issued land before the CTA may exit
+            if (it > 0) mbar_wait_bounded(&bar[kQFull], (uint32_t)((it - 1) & 1), err);
+            for (int64_t x = g - kStages; x < g; x++) {
+                if (x < 0) continue;
+                const int s = (int)(x & 1);
+                mbar_wait_bounded(&bar[kKFull + s], (uint32_t)((x >> 1) & 1), err);
+                mbar_wait_bounded(&bar[kVFull + s], (uint32_t)((x >> 1) & 1), err);
+            }
+        }
+    } else if (warp == 1) {
+        // ===================== MMA issue =====================
+        if (lane == 0) {
+            const uint32_t id_qk = instr_desc(false), id_pv = instr_desc(true);
+            const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV),
+                           aP = smem_addr(sP);
+            const uint32_t tS = tmem, tO = tmem + kBN;
+            int64_t it = 0, g = 0;
+            bool issued = false;
+            auto pv = [&](int64_t gp, bool first_of_item) -> bool {
+                const int s = (int)(gp & 1);
+                if (!wait_bar(&bar[kPFull], (uint32_t)(gp & 1), abort, err)) return false;
+                if (!wait_bar(&bar[kVFull + s], (uint32_t)((gp >> 1) & 1), abort, err)) return false;
+                tc_fence_after();
+                for (int kk = 0; kk < kBN / 16; kk++) {
+                    const uint32_t ko = (uint32_t)((kk >> 2) * kHalf + (kk & 3) * 32);
+                    const uint32_t vo = (uint32_t)(s * kTileBytes + kk * 16 * 128);
+                    umma(tO, smem_desc(aP + ko, 16, 1024), smem_desc(aV + vo, kHalf, 1024), id_pv,
+                         (first_of_item && kk == 0) ? 0u : 1u);
+                }
+                umma_commit(&bar[kOFull]);
+                umma_commit(&bar[kKvEmpty + s]);
+                issued = true;
+                return true;
+            };
+            for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
+                const Item item = item_at(k, tiles_max, B, H_q, tab);
+                if (!item.valid) continue;
+                const Req &q = tab[item.b];
+                const int64_t t0 = (int64_t)item.i * kBM;
+                const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
+                const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
+                if (!wait_bar(&bar[kQFull], (uint32_t)(it & 1), abort, err)) break;
+                bool stop = false;
+                for (int j = 0; j < n_kt; j++, g++) {
+                    const int s = (int)(g & 1);
+                    if (!wait_bar(&bar[kKFull + s], (uint32_t)((g >> 1) & 1), abort, err) ||
+                        (g > 0 && !wait_bar(&bar[kSFree], (uint32_t)((g - 1) & 1), abort, err))) {
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    for (int kk = 0; kk < kD / 16; kk++) {
+                        const uint32_t ko = (uint32_t)((kk >> 2) * kHalf + (kk & 3) * 32);
+                        umma(tS, smem_desc(aQ + ko, 16, 1024),
+                             smem_desc(aK + s * kTileBytes + ko, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
+                    }
+                    umma_commit(&bar[kSFull]);
+                    // the query tile is free once the item's last Q K^T is done
+                    if (j == n_kt - 1) umma_commit(&bar[kQEmpty]);
+                    issued = true;
+                    if (j > 0 && !pv(g - 1, j == 1)) {
+                        stop = true;
+                        break;
+                    }
+                }
+                if (stop || !pv(g - 1, n_kt == 1)) break;
+                ++it;
+            }
+            if (issued) {  // every MMA issued has completed before TMEM is freed
+                umma_commit(&bar[kDrain]);
+                mbar_wait_bounded(&bar[kDrain], 0, err);
+            }
+        }
+    } else {
+        // ===================== softmax: one query row per thread ==========
+        const int quarter = warp & 3;         // TMEM lanes 32*quarter .. +31
+        const int r = quarter * 32 + lane;    // the row of the tile
+        const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
+        const uint32_t tS = tmem + lanes, tO = tmem + lanes + kBN;
+        int64_t g = 0;
+        bool stop = false;
+        for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
+            const Item item = item_at(k, tiles_max, B, H_q, tab);
+            if (!item.valid) continue;
+            const Req &q = tab[item.b];
+            const int64_t t0 = (int64_t)item.i * kBM;
+            const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
+            const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
+            const int n_full = (int)((pi_of(q, t0, w) + 1) / kBN);  // tiles no row masks
+            const int64_t c = (int64_t)q.P + q.n + q.N;
+            const int64_t t = t0 + r;
+            const int64_t lim = pi_of(q, t < q.S ? t : (int64_t)q.S - 1, w);
+            float m = -INFINITY, l = 0.f;
+            for (int j = 0; j < n_kt; j++, g++) {
+                if (!__all_sync(0xffffffffu, wait_bar(&bar[kSFull], (uint32_t)(g & 1), abort, err))) {
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const bool masked = j >= n_full;
+                const int64_t e0 = (int64_t)j * kBN;
+                // pass 1: row maximum of the tile
+                float mx = -INFINITY;
+                for (int ch = 0; ch < 4; ch++) {
+                    uint32_t v[32];
+                    tmem_ld32(tS + ch * 32, v);
+#pragma unroll
+                    for (int i = 0; i < 32; i++) {
+                        float x = __uint_as_float(v[i]);
+                        if (masked && e0 + ch * 32 + i > lim) x = -INFINITY;
+                        mx = fmaxf(mx, x);
+                    }
+                }
+                const float mnew = fmaxf(m, mx * sl2);
+                // pass 2: weights p = 2^(s * sl2 - m), packed to bf16 pairs
+                float rowsum = 0.f;
+                uint32_t pk[64];
+                for (int ch = 0; ch < 4; ch++) {
+                    uint32_t v[32];
+                    tmem_ld32(tS + ch * 32, v);
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        const int64_t e = e0 + ch * 32 + i;
+                        float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mnew));
+                        float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mnew));
+                        if (masked && e > lim) p0 = 0.f;
+                        if (masked && e + 1 > lim) p1 = 0.f;
+                        rowsum += p0 + p1;
+                        __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+                        pk[ch * 16 + i / 2] = *reinterpret_cast<uint32_t *>(&h);
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(&bar[kSFree]);  // S may be overwritten by the next Q K^T
+                const float corr = fast_exp2(m - mnew);  // 0 on the first tile
+                if (j > 0) {
+                    // O holds the earlier tiles' sum (and P is free) once PV(j-1) is done
+                    if (!__all_sync(0xffffffffu,
+                                    wait_bar(&bar[kOFull], (uint32_t)((g - 1) & 1), abort, err))) {
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    if (__any_sync(0xffffffffu, mnew > m)) {
+                        for (int ch = 0; ch < 4; ch++) {
+                            uint32_t v[32];
+                            tmem_ld32(tO + ch * 32, v);
+#pragma unroll
+                            for (int i = 0; i < 32; i++)
+                                v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
+                            tmem_st32(tO + ch * 32, v);
+                        }
+                        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    }
+                }
+                l = l * corr + rowsum;
+                m = mnew;
+                if (e0 + kBN > c) {
+                    // value rows at or past the compressed length: zero them
+                    const int s = (int)(g & 1);
+                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kVFull + s], (uint32_t)((g >> 1) & 1),
+                                                          abort, err))) {
+                        stop = true;
+                        break;
+                    }
+                    if (e0 + r >= c) {
+                        unsigned char *row = sV + s * kTileBytes + r * 128;
+#pragma unroll
+                        for (int x = 0; x < 8; x++) {
+                            *reinterpret_cast<uint4 *>(row + x * 16) = make_uint4(0, 0, 0, 0);
+                            *reinterpret_cast<uint4 *>(row + kHalf + x * 16) = make_uint4(0, 0, 0, 0);
+                        }
+                    }
+                }
+                // P row r in the 128-byte swizzled K-major layout of the MMA's A operand
+#pragma unroll
+                for (int c16 = 0; c16 < 16; c16++) {
+                    unsigned char *dst =
+                        sP + (c16 >> 3) * kHalf + r * 128 + (((c16 & 7) ^ (r & 7)) * 16);
+                    *reinterpret_cast<uint4 *>(dst) =
+                        make_uint4(pk[4 * c16], pk[4 * c16 + 1], pk[4 * c16 + 2], pk[4 * c16 + 3]);
+                }
+                fence_proxy_async_shared();
+                tc_fence_before();
+                mbar_arrive(&bar[kPFull]);
+            }
+            if (stop) break;
+            // epilogue: O / l once the last PV is done
+            if (!__all_sync(0xffffffffu, wait_bar(&bar[kOFull], (uint32_t)((g - 1) & 1), abort, err)))
+                break;
+            tc_fence_after();
+            const float inv = 1.f / l;
+            __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq) * kD;
+            for (int ch = 0; ch < 4; ch++) {
+                uint32_t v[32];
+                tmem_ld32(tO + ch * 32, v);
+                if (t < q.S) {
+#pragma unroll
+                    for (int x = 0; x < 4; x++) {
+                        uint32_t wv[4];
+#pragma unroll
+                        for (int y = 0; y < 4; y++) {
+                            __nv_bfloat162 h = __floats2bfloat162_rn(
+                                __uint_as_float(v[8 * x + 2 * y]) * inv,
+                                __uint_as_float(v[8 * x + 2 * y + 1]) * inv);
+                            wv[y] = *reinterpret_cast<uint32_t *>(&h);
+                        }
+                        *reinterpret_cast<uint4 *>(dst + ch * 32 + x * 8) =
+                            make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                    }
+                }
+            }
+            tc_fence_before();
+        }
+    }
+
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(kTmemCols)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------- host --
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static std::once_flag once;
+    static EncodeTiledFn fn = nullptr;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+bool encode(CUtensorMap *m, const void *base, int rank, const cuuint64_t *dims,
+            const cuuint64_t *strides, const cuuint32_t *box) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const cuuint32_t es[3] = {1, 1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void *>(base), dims,
+              strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool prefill_supported(speechkv_dtype dtype, int d) { return dtype == SPEECHKV_BF16 && d == kD; }
+
+cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t stream) {
+    CUtensorMap tq, tk, tv;
+    {
+        const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.H_q, (cuuint64_t)a.q_rows};
+        const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.H_q * kD * 2};
+        const cuuint32_t box[3] = {64, 1, kBM};
+        if (!encode(&tq, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    {
+        const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)(a.cache_rows * a.H_kv)};
+        const cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+        const cuuint32_t box[2] = {64, kBN};
+        if (!encode(&tk, a.k_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
+        if (!encode(&tv, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
+    }
+    const size_t smem = smem_bytes(a.B);
+    static std::once_flag once;
+    static cudaError_t attr_err = cudaSuccess;
+    std::call_once(once, [] {
+        attr_err = cudaFuncSetAttribute(prefill_attn_kernel,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                        (int)smem_bytes(SPEECHKV_MAX_BATCH));
+    });
+    if (attr_err != cudaSuccess) return attr_err;
+    const float sl2 = a.scale * 1.4426950408889634f;
+    prefill_attn_kernel<<<num_sms, kThreads, smem, stream>>>(
+        tq, tk, tv, a.q_off, a.P, a.T, a.N, a.cache_off, static_cast<__nv_bfloat16 *>(a.out),
+        a.q_rows, a.cache_rows, sl2, a.B, a.H_q, a.H_kv, a.w_eff, a.err);
+    return cudaGetLastError();
+}
+
+}  // namespace speechkv

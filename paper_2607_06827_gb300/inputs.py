@@ -126,6 +126,7 @@ def qwen_ragged(B: int = 128, w: int = 4, seed: int = 1005) -> Workload:
 # --------------------------------------------------------------------------
 TAG_PREFILL_K, TAG_PREFILL_V, TAG_GATE = 1, 2, 3
 TAG_Q, TAG_KNEW, TAG_VNEW, TAG_GEN_K, TAG_GEN_V = 4, 5, 6, 7, 8
+TAG_PREFILL_Q = 9
 
 
 def rng_for(seed: int, *key: int) -> np.random.Generator:
@@ -154,6 +155,13 @@ def prefill_kv(wl: Workload, layer: int, b: int):
     k = normal_f32(wl.seed, (TAG_PREFILL_K, layer, b), shape)
     v = normal_f32(wl.seed, (TAG_PREFILL_V, layer, b), shape)
     return to_storage(k, wl.dtype), to_storage(v, wl.dtype)
+
+
+def prefill_q(wl: Workload, layer: int, b: int):
+    """Prompt queries of request b at ``layer``: [P+T+N, H_q, d]."""
+    S = wl.P[b] + wl.T[b] + wl.N[b]
+    q = normal_f32(wl.seed, (TAG_PREFILL_Q, layer, b), (S, wl.H_q, wl.d))
+    return to_storage(q, wl.dtype)
 
 
 def generated_kv(wl: Workload, layer: int, b: int):

@@ -46,6 +46,9 @@ SIGNATURES = {
                                                     _I32, _I32, _I32, _I32, _I32, _I32,
                                                     _I32, _I32, ctypes.c_int,
                                                     ctypes.c_uint32, _P]),
+    "speechkv_prefill_attn": (ctypes.c_int, [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _I64, _P, _F,
+                                             _I32, _I32, _I32, _I32, _I32, _I32, _I32,
+                                             ctypes.c_int, _P]),
     "speechkv_check_device_error": (ctypes.c_int, [_P]),
 }
 
@@ -192,6 +195,22 @@ def decode_step_noalloc(q, k_new, v_new, k_cache, v_cache, cache_off, length, ou
         _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas,
         _dtype_code(q), flags, _stream(stream)),
         "speechkv_decode_step_noalloc")
+
+
+def prefill_attn(q, q_off, P, T, N, k_cache, v_cache, cache_off, out, w: int, layer: int,
+                 l0: int, H_kv: int, scale: float = 0.0, stream=None):
+    """speechkv_prefill_attn: q/out [q_rows, H_q, d] (bf16, token-major
+    prompt queries); q_off/cache_off int64 [B+1]; P/T/N int32 [B]; the
+    caches as speechkv_pool wrote them (their element count fixes
+    cache_rows)."""
+    q_rows, H_q, d = q.shape
+    B = P.numel()
+    cache_rows = k_cache.numel() // (H_kv * d)
+    _check(load().speechkv_prefill_attn(
+        _ptr(q), _ptr(q_off), q_rows, _ptr(P), _ptr(T), _ptr(N), _ptr(k_cache), _ptr(v_cache),
+        _ptr(cache_off), cache_rows, _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0,
+        _dtype_code(q), _stream(stream)),
+        "speechkv_prefill_attn")
 
 
 def check_device_error(stream=None) -> int:

@@ -22,7 +22,7 @@ def test_header_declares_the_path():
     names = _declared()
     for n in ("speechkv_pool", "speechkv_append", "speechkv_decode_attn", "speechkv_decode_step",
               "speechkv_compressed_len", "speechkv_decode_workspace_size",
-              "speechkv_check_device_error", "speechkv_status_string"):
+              "speechkv_check_device_error", "speechkv_status_string", "speechkv_prefill_attn"):
         assert n in names
 
 
@@ -79,6 +79,18 @@ def test_host_argument_checks_without_gpu():
     assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 128, 0, 0, 0, sk.BF16, z) == sk.ERR_INVALID_ARG
     assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 80, 4, 0, 0, sk.BF16, z) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_pool(*([z] * 11), 0, 0, 8, 128, 4, 0, 0, sk.BF16, z) == sk.OK
+    # prefill attention: bf16 and d = 128 only; 32-bit tensor-copy coordinates
+    pf = lambda B, q_rows, cache_rows, H_q, H_kv, d, w, dt: (  # noqa: E731
+        z, z, q_rows, z, z, z, z, z, z, cache_rows, z, 0.0, B, H_q, H_kv, d, w, 0, 0, dt, z)
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.F32)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 64, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 0, sk.BF16)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 12, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_prefill_attn(*pf(sk.MAX_BATCH + 1, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_prefill_attn(*pf(1, 1 << 31, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 1 << 28, 16, 8, 128, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn(*pf(0, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.OK
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
 
 
 def test_workspace_size_explicit_grid():
