@@ -13,11 +13,12 @@
 //     and of 128-row key and value tiles (two stages) from the cache;
 //   * warp 1 lane 0: tcgen05.mma issue -- S = Q K^T into a 128-column TMEM
 //     buffer, O += P V into another (V as the MN-major operand);
-//   * warps 2-5: softmax, one query row per thread (= TMEM lane): two passes
-//     over S in TMEM (row maximum, then base-2 exponentials with
-//     log2(e)/sqrt(d) folded in), P written as bf16 into shared memory in
-//     the MMA's swizzled K-major layout, O rescaled in TMEM when a warp's
-//     running maximum moved, and the epilogue O / l to global memory.
+//   * warps 2-5: softmax, one query row per thread (= TMEM lane): the S row
+//     read from TMEM in one load (S is then free for the next Q K^T), row
+//     maximum, base-2 exponentials with log2(e)/sqrt(d) folded in, P written
+//     as bf16 into shared memory in the MMA's swizzled K-major layout, O
+//     rescaled in TMEM only when a row's maximum rose by more than 2^8
+//     (lazy rescaling), and the epilogue O / l to global memory.
 // Cache rows past a request's compressed length are zeroed in the value
 // stage (their contents are unspecified and the MMA would multiply them by
 // zero weights: 0 x NaN is NaN).  Every wait is bounded; on a timeout the CTA
@@ -103,33 +104,20 @@ __device__ __forceinline__ void tc_fence_before() {
 __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
-// 32 consecutive fp32 columns of this thread's TMEM lane.
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+// All 128 fp32 columns of this thread's TMEM lane in one load.
+__device__ __forceinline__ void tmem_ld128(uint32_t taddr, uint32_t (&r)[128]) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
-          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
-          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
-          "=r"(r[31])
+        "tcgen05.ld.sync.aligned.32x32b.x128.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65,%66,%67,%68,%69,%70,%71,%72,%73,%74,%75,%76,%77,%78,%79,%80,%81,%82,%83,%84,%85,%86,%87,%88,%89,%90,%91,%92,%93,%94,%95,%96,%97,%98,%99,%100,%101,%102,%103,%104,%105,%106,%107,%108,%109,%110,%111,%112,%113,%114,%115,%116,%117,%118,%119,%120,%121,%122,%123,%124,%125,%126,%127}, [%128];"
+        : "=r"(r[0]),"=r"(r[1]),"=r"(r[2]),"=r"(r[3]),"=r"(r[4]),"=r"(r[5]),"=r"(r[6]),"=r"(r[7]),"=r"(r[8]),"=r"(r[9]),"=r"(r[10]),"=r"(r[11]),"=r"(r[12]),"=r"(r[13]),"=r"(r[14]),"=r"(r[15]),"=r"(r[16]),"=r"(r[17]),"=r"(r[18]),"=r"(r[19]),"=r"(r[20]),"=r"(r[21]),"=r"(r[22]),"=r"(r[23]),"=r"(r[24]),"=r"(r[25]),"=r"(r[26]),"=r"(r[27]),"=r"(r[28]),"=r"(r[29]),"=r"(r[30]),"=r"(r[31]),"=r"(r[32]),"=r"(r[33]),"=r"(r[34]),"=r"(r[35]),"=r"(r[36]),"=r"(r[37]),"=r"(r[38]),"=r"(r[39]),"=r"(r[40]),"=r"(r[41]),"=r"(r[42]),"=r"(r[43]),"=r"(r[44]),"=r"(r[45]),"=r"(r[46]),"=r"(r[47]),"=r"(r[48]),"=r"(r[49]),"=r"(r[50]),"=r"(r[51]),"=r"(r[52]),"=r"(r[53]),"=r"(r[54]),"=r"(r[55]),"=r"(r[56]),"=r"(r[57]),"=r"(r[58]),"=r"(r[59]),"=r"(r[60]),"=r"(r[61]),"=r"(r[62]),"=r"(r[63]),"=r"(r[64]),"=r"(r[65]),"=r"(r[66]),"=r"(r[67]),"=r"(r[68]),"=r"(r[69]),"=r"(r[70]),"=r"(r[71]),"=r"(r[72]),"=r"(r[73]),"=r"(r[74]),"=r"(r[75]),"=r"(r[76]),"=r"(r[77]),"=r"(r[78]),"=r"(r[79]),"=r"(r[80]),"=r"(r[81]),"=r"(r[82]),"=r"(r[83]),"=r"(r[84]),"=r"(r[85]),"=r"(r[86]),"=r"(r[87]),"=r"(r[88]),"=r"(r[89]),"=r"(r[90]),"=r"(r[91]),"=r"(r[92]),"=r"(r[93]),"=r"(r[94]),"=r"(r[95]),"=r"(r[96]),"=r"(r[97]),"=r"(r[98]),"=r"(r[99]),"=r"(r[100]),"=r"(r[101]),"=r"(r[102]),"=r"(r[103]),"=r"(r[104]),"=r"(r[105]),"=r"(r[106]),"=r"(r[107]),"=r"(r[108]),"=r"(r[109]),"=r"(r[110]),"=r"(r[111]),"=r"(r[112]),"=r"(r[113]),"=r"(r[114]),"=r"(r[115]),"=r"(r[116]),"=r"(r[117]),"=r"(r[118]),"=r"(r[119]),"=r"(r[120]),"=r"(r[121]),"=r"(r[122]),"=r"(r[123]),"=r"(r[124]),"=r"(r[125]),"=r"(r[126]),"=r"(r[127])
         : "r"(taddr));
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+__device__ __forceinline__ void tmem_st128(uint32_t taddr, const uint32_t (&r)[128]) {
     asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
-        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
-            taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
-        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
-        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
-        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
-        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        "tcgen05.st.sync.aligned.32x32b.x128.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64,%65,%66,%67,%68,%69,%70,%71,%72,%73,%74,%75,%76,%77,%78,%79,%80,%81,%82,%83,%84,%85,%86,%87,%88,%89,%90,%91,%92,%93,%94,%95,%96,%97,%98,%99,%100,%101,%102,%103,%104,%105,%106,%107,%108,%109,%110,%111,%112,%113,%114,%115,%116,%117,%118,%119,%120,%121,%122,%123,%124,%125,%126,%127,%128};"
+        :: "r"(taddr), "r"(r[0]),"r"(r[1]),"r"(r[2]),"r"(r[3]),"r"(r[4]),"r"(r[5]),"r"(r[6]),"r"(r[7]),"r"(r[8]),"r"(r[9]),"r"(r[10]),"r"(r[11]),"r"(r[12]),"r"(r[13]),"r"(r[14]),"r"(r[15]),"r"(r[16]),"r"(r[17]),"r"(r[18]),"r"(r[19]),"r"(r[20]),"r"(r[21]),"r"(r[22]),"r"(r[23]),"r"(r[24]),"r"(r[25]),"r"(r[26]),"r"(r[27]),"r"(r[28]),"r"(r[29]),"r"(r[30]),"r"(r[31]),"r"(r[32]),"r"(r[33]),"r"(r[34]),"r"(r[35]),"r"(r[36]),"r"(r[37]),"r"(r[38]),"r"(r[39]),"r"(r[40]),"r"(r[41]),"r"(r[42]),"r"(r[43]),"r"(r[44]),"r"(r[45]),"r"(r[46]),"r"(r[47]),"r"(r[48]),"r"(r[49]),"r"(r[50]),"r"(r[51]),"r"(r[52]),"r"(r[53]),"r"(r[54]),"r"(r[55]),"r"(r[56]),"r"(r[57]),"r"(r[58]),"r"(r[59]),"r"(r[60]),"r"(r[61]),"r"(r[62]),"r"(r[63]),"r"(r[64]),"r"(r[65]),"r"(r[66]),"r"(r[67]),"r"(r[68]),"r"(r[69]),"r"(r[70]),"r"(r[71]),"r"(r[72]),"r"(r[73]),"r"(r[74]),"r"(r[75]),"r"(r[76]),"r"(r[77]),"r"(r[78]),"r"(r[79]),"r"(r[80]),"r"(r[81]),"r"(r[82]),"r"(r[83]),"r"(r[84]),"r"(r[85]),"r"(r[86]),"r"(r[87]),"r"(r[88]),"r"(r[89]),"r"(r[90]),"r"(r[91]),"r"(r[92]),"r"(r[93]),"r"(r[94]),"r"(r[95]),"r"(r[96]),"r"(r[97]),"r"(r[98]),"r"(r[99]),"r"(r[100]),"r"(r[101]),"r"(r[102]),"r"(r[103]),"r"(r[104]),"r"(r[105]),"r"(r[106]),"r"(r[107]),"r"(r[108]),"r"(r[109]),"r"(r[110]),"r"(r[111]),"r"(r[112]),"r"(r[113]),"r"(r[114]),"r"(r[115]),"r"(r[116]),"r"(r[117]),"r"(r[118]),"r"(r[119]),"r"(r[120]),"r"(r[121]),"r"(r[122]),"r"(r[123]),"r"(r[124]),"r"(r[125]),"r"(r[126]),"r"(r[127])
         : "memory");
 }
-
 // TMA tensor copies global -> shared (completion as transaction bytes on bar)
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x, int y,
                                        uint64_t *bar) {
@@ -406,40 +394,44 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const bool masked = j >= n_full;
                 const int64_t e0 = (int64_t)j * kBN;
-                // pass 1: row maximum of the tile
+                // keys e0 + i, i <= vis, are visible to this row
+                int64_t vis64 = lim - e0;
+                vis64 = vis64 > kBN - 1 ? kBN - 1 : (vis64 < -1 ? -1 : vis64);
+                const int vis = masked ? (int)vis64 : kBN - 1;
+                uint32_t v[128];
+                tmem_ld128(tS, v);
+                tc_fence_before();
+                mbar_arrive(&bar[kSFree]);  // S is in registers: the next Q K^T may overwrite it
                 float mx = -INFINITY;
-                for (int ch = 0; ch < 4; ch++) {
-                    uint32_t v[32];
-                    tmem_ld32(tS + ch * 32, v);
+                if (masked) {
 #pragma unroll
-                    for (int i = 0; i < 32; i++) {
-                        float x = __uint_as_float(v[i]);
-                        if (masked && e0 + ch * 32 + i > lim) x = -INFINITY;
-                        mx = fmaxf(mx, x);
-                    }
+                    for (int i = 0; i < kBN; i++)
+                        mx = fmaxf(mx, i <= vis ? __uint_as_float(v[i]) : -INFINITY);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < kBN; i++) mx = fmaxf(mx, __uint_as_float(v[i]));
                 }
-                const float mnew = fmaxf(m, mx * sl2);
-                // pass 2: weights p = 2^(s * sl2 - m), packed to bf16 pairs
+                mx *= sl2;
+                // Lazy rescaling: the weights keep using the running maximum
+                // unless the tile's exceeds it by more than 8 (weights then
+                // stay below 2^8); O / l is the same either way.
+                const bool bump = mx > m + 8.f;  // always on the first tile (m = -inf)
+                const float mu = bump ? mx : m;
+                const float corr = fast_exp2(m - mu);  // 1 without a bump, 0 on the first tile
                 float rowsum = 0.f;
                 uint32_t pk[64];
-                for (int ch = 0; ch < 4; ch++) {
-                    uint32_t v[32];
-                    tmem_ld32(tS + ch * 32, v);
 #pragma unroll
-                    for (int i = 0; i < 32; i += 2) {
-                        const int64_t e = e0 + ch * 32 + i;
-                        float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mnew));
-                        float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mnew));
-                        if (masked && e > lim) p0 = 0.f;
-                        if (masked && e + 1 > lim) p1 = 0.f;
-                        rowsum += p0 + p1;
-                        __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-                        pk[ch * 16 + i / 2] = *reinterpret_cast<uint32_t *>(&h);
+                for (int i = 0; i < kBN; i += 2) {
+                    float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mu));
+                    float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mu));
+                    if (masked) {
+                        p0 = i <= vis ? p0 : 0.f;
+                        p1 = i + 1 <= vis ? p1 : 0.f;
                     }
+                    rowsum += p0 + p1;
+                    __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
+                    pk[i / 2] = *reinterpret_cast<uint32_t *>(&h);
                 }
-                tc_fence_before();
-                mbar_arrive(&bar[kSFree]);  // S may be overwritten by the next Q K^T
-                const float corr = fast_exp2(m - mnew);  // 0 on the first tile
                 if (j > 0) {
                     // O holds the earlier tiles' sum (and P is free) once PV(j-1) is done
                     if (!__all_sync(0xffffffffu,
@@ -448,20 +440,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
-                    if (__any_sync(0xffffffffu, mnew > m)) {
-                        for (int ch = 0; ch < 4; ch++) {
-                            uint32_t v[32];
-                            tmem_ld32(tO + ch * 32, v);
+                    if (__any_sync(0xffffffffu, bump)) {
+                        uint32_t o[128];
+                        tmem_ld128(tO, o);
 #pragma unroll
-                            for (int i = 0; i < 32; i++)
-                                v[i] = __float_as_uint(__uint_as_float(v[i]) * corr);
-                            tmem_st32(tO + ch * 32, v);
-                        }
+                        for (int i = 0; i < 128; i++)
+                            o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
+                        tmem_st128(tO, o);
                         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                     }
                 }
                 l = l * corr + rowsum;
-                m = mnew;
+                m = mu;
                 if (e0 + kBN > c) {
                     // value rows at or past the compressed length: zero them
                     const int s = (int)(g & 1);
@@ -498,23 +488,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             const float inv = 1.f / l;
             __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq) * kD;
-            for (int ch = 0; ch < 4; ch++) {
-                uint32_t v[32];
-                tmem_ld32(tO + ch * 32, v);
-                if (t < q.S) {
+            uint32_t o[128];
+            tmem_ld128(tO, o);
+            if (t < q.S) {
 #pragma unroll
-                    for (int x = 0; x < 4; x++) {
-                        uint32_t wv[4];
+                for (int x = 0; x < 16; x++) {
+                    uint32_t wv[4];
 #pragma unroll
-                        for (int y = 0; y < 4; y++) {
-                            __nv_bfloat162 h = __floats2bfloat162_rn(
-                                __uint_as_float(v[8 * x + 2 * y]) * inv,
-                                __uint_as_float(v[8 * x + 2 * y + 1]) * inv);
-                            wv[y] = *reinterpret_cast<uint32_t *>(&h);
-                        }
-                        *reinterpret_cast<uint4 *>(dst + ch * 32 + x * 8) =
-                            make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                    for (int y = 0; y < 4; y++) {
+                        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(o[8 * x + 2 * y]) * inv,
+                                                                 __uint_as_float(o[8 * x + 2 * y + 1]) * inv);
+                        wv[y] = *reinterpret_cast<uint32_t *>(&h);
                     }
+                    *reinterpret_cast<uint4 *>(dst + x * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
                 }
             }
             tc_fence_before();
