@@ -14,12 +14,12 @@ d = 128), bf16, batch 8, 20 min of audio (15000 frames at 80 ms), w = 4,
 64-token prompt, 64 tokens already generated (mid-run of a 128-token
 decode).  Also reported: the same workload uncompressed (w = 1, identical
 seeded inputs), a sweep over 2/5/10/20 min with w in {4, 8}, an end-to-end
-number through the C ABI with host buffers, and the CPU oracle timed on the
-host cores.
+number through the C ABI with host buffers, the CPU oracle timed on the host
+cores, and the prefill attention (speechkv_prefill_attn, tensor cores) over
+the whole prompt of the batch at a pooled and a full-resolution layer.
 
 Timed steps run as CUDA graphs (chunks of steps captured ahead of the timed
-region), with CUDA events around every decode-attention launch recorded
-inside the graphs.  Consecutive layers read disjoint caches and the per-step
+region), timed with CUDA events around the graph replays.  Consecutive layers read disjoint caches and the per-step
 working set (several GB) exceeds the 129 MB L2, so no explicit flush is
 needed.
 
@@ -47,6 +47,7 @@ UNIT = "us/step/layer"
 HEADLINE_MINUTES, HEADLINE_W, GENERATED = 20, 4, 64
 SWEEP = [(2, 4), (2, 8), (5, 4), (5, 8), (10, 4), (10, 8), (20, 8)]
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "decode_attn_traffic.txt")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_06827_gb300", "csrc", f)
                   for f in ("decode_attn.cu", "common.cuh")]
@@ -68,6 +69,10 @@ def parse_args():
     ap.add_argument("--no-unfused", action="store_true",
                     help="skip timing append + decode_attn as two launches")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true",
+                    help="skip the prefill-attention measurement")
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="diagnostic: time only the prefill attention and print its section")
     ap.add_argument("--cpu-seconds", type=float, default=12.0,
                     help="budget of the oracle CPU baseline sample")
     ap.add_argument("--graph-chunk", type=int, default=32)
@@ -462,6 +467,78 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
             "d2h_bytes_per_step": d2h, "steps": steps, "outputs_finite": ok}
 
 
+def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
+    """speechkv_prefill_attn over the whole prompt of the batch, at a pooled
+    layer (l0) and at a full-resolution one (0): CUDA-event time of one launch
+    (median of `repeats`), algorithmic FLOPs (4 d per visible query-key pair:
+    QK^T and PV) and the fraction of the measured bf16 tensor peak (burst:
+    the kernel is timed alone)."""
+    import numpy as np
+    import torch
+    from paper_2607_06827_gb300 import inputs, speechkv as sk
+    res = {}
+    S = sum(wl.full_rows())
+    off = np.zeros(wl.B + 1, dtype=np.int64)
+    off[1:] = np.cumsum(wl.full_rows())
+    q_off = torch.from_numpy(off).cuda()
+    t32 = lambda x: torch.tensor(x, dtype=torch.int32, device="cuda")  # noqa: E731
+    P, T, N = t32(wl.P), t32(wl.T), t32(wl.N)
+    q = inputs.device_normal((S, wl.H_q, wl.d), torch.bfloat16, "cuda", wl.seed, 40)
+    out = torch.empty_like(q)
+    for kind, layer in (("pooled_layer", wl.l0), ("full_layer", 0)):
+        w_eff = wl.w if layer >= wl.l0 else 1
+        cap = [sk.compressed_len(p, t, n, 0, wl.w, layer, wl.l0)
+               for p, t, n in zip(wl.P, wl.T, wl.N)]
+        coff = np.zeros(wl.B + 1, dtype=np.int64)
+        coff[1:] = np.cumsum(cap)
+        rows = int(coff[-1])
+        kc = inputs.device_normal((rows * wl.H_kv * wl.d,), torch.bfloat16, "cuda", wl.seed, 41, layer)
+        vc = inputs.device_normal((rows * wl.H_kv * wl.d,), torch.bfloat16, "cuda", wl.seed, 42, layer)
+        cache_off = torch.from_numpy(coff).cuda()
+        # visible (query, key) pairs: query t sees compressed rows 0 .. pi(t)
+        pairs = 0
+        for p_, t_, n_ in zip(wl.P, wl.T, wl.N):
+            n = -(-t_ // w_eff)
+            t = np.arange(p_ + t_ + n_, dtype=np.int64)
+            pi = np.where(t < p_, t, np.where(t < p_ + t_, p_ + (t - p_) // w_eff, t - t_ + n))
+            pairs += int((pi + 1).sum())
+        flops = 4.0 * wl.d * wl.H_q * pairs
+
+        def launch():
+            sk.prefill_attn(q, q_off, P, T, N, kc, vc, cache_off, out, wl.w, layer, wl.l0,
+                            wl.H_kv)
+        for _ in range(warmup):
+            launch()
+        torch.cuda.synchronize()
+        times = []
+        t0 = time.time()
+        for _ in range(repeats):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            launch()
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        clocks and clocks.mark(t0, time.time())
+        status = sk.check_device_error()
+        assert status == sk.OK, sk.status_string(status)
+        assert bool(torch.isfinite(out.float()).all())
+        ms = sorted(times)[len(times) // 2]
+        res[kind] = {"layer": layer, "w_eff": w_eff, "us": round(ms * 1e3, 1),
+                     "tflop": round(flops / 1e12, 4),
+                     "tflops": round(flops / (ms * 1e-3) / 1e12, 1)}
+        del kc, vc
+    del q, out
+    torch.cuda.empty_cache()
+    peak, kind = measured_bf16_peak()
+    for r in res.values():
+        r["frac"] = round(r["tflops"] / peak, 4)
+    res.update({"bound": "tensor", "peak": peak, "peak_kind": kind, "unit": "TFLOP/s",
+                "kernel": "prefill_attn_kernel (tcgen05, bf16, d=128): speechkv_prefill_attn",
+                "workload": f"whole prompt of the batch ({S} query rows x {wl.H_q} heads)"})
+    return res
+
+
 # ---------------------------------------------------------------------------
 # CPU oracle timing (cpu_baseline and --impl reference)
 # ---------------------------------------------------------------------------
@@ -592,6 +669,15 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+def measured_bf16_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured (burst)"
+    except (OSError, ValueError, KeyError):
+        return FALLBACK_BF16_TFLOPS, "fallback"
+
+
 def kernel_hash() -> str:
     h = hashlib.sha256()
     for p in KERNEL_SOURCES:
@@ -638,6 +724,13 @@ def main():
 
     layers = [int(x) for x in args.layers.split(",")] if args.layers else None
     wl = inputs.qwen_long_audio(args.minutes, args.w, generated=GENERATED)
+    if args.prefill_only:
+        pre = measure_prefill(inputs.qwen_long_audio(args.minutes, args.w), clocks)
+        if dist.rank == 0:
+            print(json.dumps(finite_json({"prefill": pre, "clocks": clocks.finish() if clocks
+                                          else None})), flush=True)
+        dist.close()
+        return
     main_res = measure(wl, args.steps, args.warmup, args.graph_chunk, dist, clocks, seed_key=0,
                        layers=layers)
     w1_res = None
@@ -684,6 +777,9 @@ def main():
                 "speedup_vs_w1_step": (round(w1["step_us"] / r["step_us"], 3) if w1 else None),
             })
 
+    prefill = None
+    if not args.no_prefill:
+        prefill = measure_prefill(inputs.qwen_long_audio(args.minutes, args.w), clocks)
     cpu = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args.cpu_seconds)
@@ -740,6 +836,7 @@ def main():
                 "decode_step_28_layers": round(w1_res["step_us"] / main_res["step_us"], 3),
             } if w1_res else None),
             "by_audio_len": sweep or None,
+            "prefill": prefill,
         }
         print(json.dumps(finite_json(line)), flush=True)
     dist.close()

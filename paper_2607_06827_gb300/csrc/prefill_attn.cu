@@ -8,7 +8,8 @@
 //
 // Blackwell tensor-core flash attention, bf16 in, fp32 accumulate, d = 128:
 //   * persistent: one CTA per SM walks work items (request, query head,
-//     128-row query tile), heaviest tiles (latest prompt positions) first;
+//     128-row query tile) ordered by (request, KV head), so that the CTAs
+//     running together read the same keys and values (from L2);
 //   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the query tile
 //     and of 128-row key and value tiles (two stages) from the cache;
 //   * warp 1 lane 0: tcgen05.mma issue -- S = Q K^T into a 128-column TMEM
@@ -154,20 +155,24 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatil
     }
 }
 
-// Work item k of the CTA-independent order: query tile i (from the last
-// tile of the longest request down), then request, then query head.
+// Work item k of the CTA-independent order: (request, KV head) outermost,
+// then query tiles from the last down, then the query heads of the KV head's
+// group.  CTAs working at the same time share one (request, KV head)'s keys
+// and values, which stay in L2 while they are read again and again.
 struct Item {
     int b, hq, i;
     bool valid;
 };
-__device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int B, int H_q,
+__device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int B, int H_q, int H_kv,
                                         const Req *tab) {
     Item it;
-    const int64_t per = (int64_t)B * H_q;
-    it.i = tiles_max - 1 - (int)(k / per);
-    const int rem = (int)(k % per);
-    it.b = rem / H_q;
-    it.hq = rem - it.b * H_q;
+    const int G = H_q / H_kv;
+    const int64_t per = (int64_t)tiles_max * G;  // items of one (request, KV head)
+    const int bh = (int)(k / per);
+    const int rem = (int)(k - (int64_t)bh * per);
+    it.b = bh / H_kv;
+    it.hq = (bh - it.b * H_kv) * G + rem % G;
+    it.i = tiles_max - 1 - rem / G;
     it.valid = it.i < tab[it.b].tiles;
     return it;
 }
@@ -263,7 +268,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             int64_t it = 0, g = 0;
             for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
-                const Item item = item_at(k, tiles_max, B, H_q, tab);
+                const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
                 if (!item.valid) continue;
                 const Req &q = tab[item.b];
                 const int64_t t0 = (int64_t)item.i * kBM;
@@ -328,7 +333,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 return true;
             };
             for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
-                const Item item = item_at(k, tiles_max, B, H_q, tab);
+                const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
                 if (!item.valid) continue;
                 const Req &q = tab[item.b];
                 const int64_t t0 = (int64_t)item.i * kBM;
@@ -375,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int64_t g = 0;
         bool stop = false;
         for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
-            const Item item = item_at(k, tiles_max, B, H_q, tab);
+            const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
             if (!item.valid) continue;
             const Req &q = tab[item.b];
             const int64_t t0 = (int64_t)item.i * kBM;
