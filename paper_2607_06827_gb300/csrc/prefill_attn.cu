@@ -13,13 +13,14 @@
 //   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the query tile
 //     and of 128-row key and value tiles (two stages) from the cache;
 //   * warp 1 lane 0: tcgen05.mma issue -- S = Q K^T into a 128-column TMEM
-//     buffer, O += P V into another (V as the MN-major operand);
+//     buffer, O += P V into another, with P read from TMEM (two 64-column
+//     buffers) and V as the MN-major shared-memory operand;
 //   * warps 2-5: softmax, one query row per thread (= TMEM lane): the S row
 //     read from TMEM in one load (S is then free for the next Q K^T), row
-//     maximum, base-2 exponentials with log2(e)/sqrt(d) folded in, P written
-//     as bf16 into shared memory in the MMA's swizzled K-major layout, O
-//     rescaled in TMEM only when a row's maximum rose by more than 2^8
-//     (lazy rescaling), and the epilogue O / l to global memory.
+//     maximum, base-2 exponentials with log2(e)/sqrt(d) folded in, P stored
+//     as bf16 pairs into its TMEM buffer, O rescaled in TMEM only when a
+//     row's maximum rose by more than 2^8 (lazy rescaling), and the epilogue
+//     O / l to global memory.
 // Cache rows past a request's compressed length are zeroed in the value
 // stage (their contents are unspecified and the MMA would multiply them by
 // zero weights: 0 x NaN is NaN).  Every wait is bounded; on a timeout the CTA
@@ -42,16 +43,18 @@ constexpr int kThreads = 192;
 constexpr int kTileBytes = kBM * kD * 2;  // one bf16 tile of 128 rows x 128
 constexpr int kHalf = kTileBytes / 2;     // its 64-column block (128-byte rows)
 constexpr int kStages = 2;                // key/value ring
-constexpr uint32_t kTmemCols = 256;       // S: columns 0..127, O: 128..255
+constexpr uint32_t kTmemCols = 512;       // S: 0..127, O: 128..255, P: 256..319 and 320..383
 
 // shared memory (offsets from a 1024-byte aligned base)
 constexpr int kOffQ = 0;
 constexpr int kOffK = kOffQ + kTileBytes;
 constexpr int kOffV = kOffK + kStages * kTileBytes;
-constexpr int kOffP = kOffV + kStages * kTileBytes;
-constexpr int kOffBar = kOffP + kTileBytes;
-enum Bar { kQFull, kQEmpty, kKFull, kVFull = kKFull + kStages, kKvEmpty = kVFull + kStages,
-           kSFull = kKvEmpty + kStages, kSFree, kPFull, kOFull, kDrain, kNumBars };
+constexpr int kOffBar = kOffV + kStages * kTileBytes;
+enum Bar { kQFull, kQEmpty, kKFull, kVFull = kKFull + kStages, kKEmpty = kVFull + kStages,
+           kVEmpty = kKEmpty + kStages, kSFull = kVEmpty + kStages, kSFree,
+           kPFull,                // [2]: P of tile g is in TMEM buffer g & 1
+           kPFree = kPFull + 2,   // [2]: the P V that read buffer g & 1 is done
+           kDrain = kPFree + 2, kNumBars };
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem address, abort flag, largest tile count
 constexpr int kOffTab = kOffMisc + 16;
 
@@ -91,6 +94,15 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(id), "r"(accumulate));
 }
+// The same with the A operand in TMEM: row m in lane m, two bf16 per 32-bit
+// column (the even element in the low half), 8 columns per 16-element K step.
+__device__ __forceinline__ void umma_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                            uint32_t id, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(id), "r"(accumulate));
+}
 // Arrive on `bar` once every tcgen05 operation issued so far by this thread
 // has completed.
 __device__ __forceinline__ void umma_commit(uint64_t *bar) {
@@ -119,6 +131,15 @@ __device__ __forceinline__ void tmem_st128(uint32_t taddr, const uint32_t (&r)[1
         :: "r"(taddr), "r"(r[0]),"r"(r[1]),"r"(r[2]),"r"(r[3]),"r"(r[4]),"r"(r[5]),"r"(r[6]),"r"(r[7]),"r"(r[8]),"r"(r[9]),"r"(r[10]),"r"(r[11]),"r"(r[12]),"r"(r[13]),"r"(r[14]),"r"(r[15]),"r"(r[16]),"r"(r[17]),"r"(r[18]),"r"(r[19]),"r"(r[20]),"r"(r[21]),"r"(r[22]),"r"(r[23]),"r"(r[24]),"r"(r[25]),"r"(r[26]),"r"(r[27]),"r"(r[28]),"r"(r[29]),"r"(r[30]),"r"(r[31]),"r"(r[32]),"r"(r[33]),"r"(r[34]),"r"(r[35]),"r"(r[36]),"r"(r[37]),"r"(r[38]),"r"(r[39]),"r"(r[40]),"r"(r[41]),"r"(r[42]),"r"(r[43]),"r"(r[44]),"r"(r[45]),"r"(r[46]),"r"(r[47]),"r"(r[48]),"r"(r[49]),"r"(r[50]),"r"(r[51]),"r"(r[52]),"r"(r[53]),"r"(r[54]),"r"(r[55]),"r"(r[56]),"r"(r[57]),"r"(r[58]),"r"(r[59]),"r"(r[60]),"r"(r[61]),"r"(r[62]),"r"(r[63]),"r"(r[64]),"r"(r[65]),"r"(r[66]),"r"(r[67]),"r"(r[68]),"r"(r[69]),"r"(r[70]),"r"(r[71]),"r"(r[72]),"r"(r[73]),"r"(r[74]),"r"(r[75]),"r"(r[76]),"r"(r[77]),"r"(r[78]),"r"(r[79]),"r"(r[80]),"r"(r[81]),"r"(r[82]),"r"(r[83]),"r"(r[84]),"r"(r[85]),"r"(r[86]),"r"(r[87]),"r"(r[88]),"r"(r[89]),"r"(r[90]),"r"(r[91]),"r"(r[92]),"r"(r[93]),"r"(r[94]),"r"(r[95]),"r"(r[96]),"r"(r[97]),"r"(r[98]),"r"(r[99]),"r"(r[100]),"r"(r[101]),"r"(r[102]),"r"(r[103]),"r"(r[104]),"r"(r[105]),"r"(r[106]),"r"(r[107]),"r"(r[108]),"r"(r[109]),"r"(r[110]),"r"(r[111]),"r"(r[112]),"r"(r[113]),"r"(r[114]),"r"(r[115]),"r"(r[116]),"r"(r[117]),"r"(r[118]),"r"(r[119]),"r"(r[120]),"r"(r[121]),"r"(r[122]),"r"(r[123]),"r"(r[124]),"r"(r[125]),"r"(r[126]),"r"(r[127])
         : "memory");
 }
+// 64 32-bit columns of this thread's TMEM lane (then waits for the store).
+__device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&r)[64]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63,%64};"
+        :: "r"(taddr), "r"(r[0]),"r"(r[1]),"r"(r[2]),"r"(r[3]),"r"(r[4]),"r"(r[5]),"r"(r[6]),"r"(r[7]),"r"(r[8]),"r"(r[9]),"r"(r[10]),"r"(r[11]),"r"(r[12]),"r"(r[13]),"r"(r[14]),"r"(r[15]),"r"(r[16]),"r"(r[17]),"r"(r[18]),"r"(r[19]),"r"(r[20]),"r"(r[21]),"r"(r[22]),"r"(r[23]),"r"(r[24]),"r"(r[25]),"r"(r[26]),"r"(r[27]),"r"(r[28]),"r"(r[29]),"r"(r[30]),"r"(r[31]),"r"(r[32]),"r"(r[33]),"r"(r[34]),"r"(r[35]),"r"(r[36]),"r"(r[37]),"r"(r[38]),"r"(r[39]),"r"(r[40]),"r"(r[41]),"r"(r[42]),"r"(r[43]),"r"(r[44]),"r"(r[45]),"r"(r[46]),"r"(r[47]),"r"(r[48]),"r"(r[49]),"r"(r[50]),"r"(r[51]),"r"(r[52]),"r"(r[53]),"r"(r[54]),"r"(r[55]),"r"(r[56]),"r"(r[57]),"r"(r[58]),"r"(r[59]),"r"(r[60]),"r"(r[61]),"r"(r[62]),"r"(r[63])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // TMA tensor copies global -> shared (completion as transaction bytes on bar)
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *map, int x, int y,
                                        uint64_t *bar) {
@@ -204,12 +225,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int s = 0; s < kStages; s++) {
             mbar_init(&bar[kKFull + s], 1);
             mbar_init(&bar[kVFull + s], 1);
-            mbar_init(&bar[kKvEmpty + s], 1);
+            mbar_init(&bar[kKEmpty + s], 1);
+            mbar_init(&bar[kVEmpty + s], 1);
         }
         mbar_init(&bar[kSFull], 1);
         mbar_init(&bar[kSFree], kBM);
-        mbar_init(&bar[kPFull], kBM);
-        mbar_init(&bar[kOFull], 1);
+        for (int x = 0; x < 2; x++) {
+            mbar_init(&bar[kPFull + x], kBM);
+            mbar_init(&bar[kPFree + x], 1);
+        }
         mbar_init(&bar[kDrain], 1);
         fence_mbar_init();
         *abort = 0;
@@ -261,12 +285,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tiles_max = *tiles_max_s;
     const int64_t total = (int64_t)tiles_max * B * H_q;
 
-    unsigned char *sQ = sm + kOffQ, *sK = sm + kOffK, *sV = sm + kOffV, *sP = sm + kOffP;
+    unsigned char *sQ = sm + kOffQ, *sK = sm + kOffK, *sV = sm + kOffV;
 
     if (warp == 0) {
         // ===================== TMA producer =====================
         if (lane == 0) {
             int64_t it = 0, g = 0;
+            bool k_only = false;
             for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
                 const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
                 if (!item.valid) continue;
@@ -283,8 +308,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bool stop = false;
                 for (int j = 0; j < n_kt; j++, g++) {
                     const int s = (int)(g & 1);
-                    if (g >= kStages &&
-                        !wait_bar(&bar[kKvEmpty + s], (uint32_t)(((g >> 1) - 1) & 1), abort, err)) {
+                    const uint32_t ph = (uint32_t)(((g >> 1) - 1) & 1);
+                    // keys are free once their Q K^T is done, values once their P V is
+                    if (g >= kStages && !wait_bar(&bar[kKEmpty + s], ph, abort, err)) {
                         stop = true;
                         break;
                     }
@@ -292,6 +318,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive_expect_tx(&bar[kKFull + s], kTileBytes);
                     tma_2d(sK + s * kTileBytes, &tm_k, 0, y, &bar[kKFull + s]);
                     tma_2d(sK + s * kTileBytes + kHalf, &tm_k, 64, y, &bar[kKFull + s]);
+                    if (g >= kStages && !wait_bar(&bar[kVEmpty + s], ph, abort, err)) {
+                        k_only = true;  // this tile's keys are in flight, its values not
+                        stop = true;
+                        break;
+                    }
                     mbar_arrive_expect_tx(&bar[kVFull + s], kTileBytes);
                     tma_2d(sV + s * kTileBytes, &tm_v, 0, y, &bar[kVFull + s]);
                     tma_2d(sV + s * kTileBytes + kHalf, &tm_v, 64, y, &bar[kVFull + s]);
@@ -306,29 +337,36 @@ __global__ void __launch_bounds__(kThreads, 1)
                 mbar_wait_bounded(&bar[kKFull + s], (uint32_t)((x >> 1) & 1), err);
                 mbar_wait_bounded(&bar[kVFull + s], (uint32_t)((x >> 1) & 1), err);
             }
+            if (k_only) mbar_wait_bounded(&bar[kKFull + (g & 1)], (uint32_t)((g >> 1) & 1), err);
         }
     } else if (warp == 1) {
         // ===================== MMA issue =====================
         if (lane == 0) {
             const uint32_t id_qk = instr_desc(false), id_pv = instr_desc(true);
-            const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV),
-                           aP = smem_addr(sP);
-            const uint32_t tS = tmem, tO = tmem + kBN;
+            const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV);
+            const uint32_t tS = tmem, tO = tmem + kBN, tP = tmem + 2 * kBN;
+            // Descriptors are built once per buffer; a K step or a stage only
+            // moves the start address, whose field (address / 16, 14 bits)
+            // cannot carry over inside shared memory.
+            const uint64_t dQ = smem_desc(aQ, 16, 1024);
+            const uint64_t dK = smem_desc(aK, 16, 1024), dV = smem_desc(aV, kHalf, 1024);
+            constexpr uint64_t kStageD = kTileBytes >> 4;
             int64_t it = 0, g = 0;
             bool issued = false;
             auto pv = [&](int64_t gp, bool first_of_item) -> bool {
                 const int s = (int)(gp & 1);
-                if (!wait_bar(&bar[kPFull], (uint32_t)(gp & 1), abort, err)) return false;
+                if (!wait_bar(&bar[kPFull + s], (uint32_t)((gp >> 1) & 1), abort, err)) return false;
                 if (!wait_bar(&bar[kVFull + s], (uint32_t)((gp >> 1) & 1), abort, err)) return false;
                 tc_fence_after();
+                const uint64_t dVs = dV + (uint64_t)s * kStageD;
+#pragma unroll
                 for (int kk = 0; kk < kBN / 16; kk++) {
-                    const uint32_t ko = (uint32_t)((kk >> 2) * kHalf + (kk & 3) * 32);
-                    const uint32_t vo = (uint32_t)(s * kTileBytes + kk * 16 * 128);
-                    umma(tO, smem_desc(aP + ko, 16, 1024), smem_desc(aV + vo, kHalf, 1024), id_pv,
-                         (first_of_item && kk == 0) ? 0u : 1u);
+                    const uint64_t vo = (uint64_t)((kk * 16 * 128) >> 4);  // 16 keys further
+                    umma_tmem_a(tO, tP + s * (kBN / 2) + kk * 8, dVs + vo, id_pv,
+                                (first_of_item && kk == 0) ? 0u : 1u);
                 }
-                umma_commit(&bar[kOFull]);
-                umma_commit(&bar[kKvEmpty + s]);
+                umma_commit(&bar[kPFree + s]);
+                umma_commit(&bar[kVEmpty + s]);
                 issued = true;
                 return true;
             };
@@ -349,12 +387,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         break;
                     }
                     tc_fence_after();
+                    const uint64_t dKs = dK + (uint64_t)s * kStageD;
+#pragma unroll
                     for (int kk = 0; kk < kD / 16; kk++) {
-                        const uint32_t ko = (uint32_t)((kk >> 2) * kHalf + (kk & 3) * 32);
-                        umma(tS, smem_desc(aQ + ko, 16, 1024),
-                             smem_desc(aK + s * kTileBytes + ko, 16, 1024), id_qk, kk > 0 ? 1u : 0u);
+                        const uint64_t ko = (uint64_t)(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
+                        umma(tS, dQ + ko, dKs + ko, id_qk, kk > 0 ? 1u : 0u);
                     }
                     umma_commit(&bar[kSFull]);
+                    umma_commit(&bar[kKEmpty + s]);
                     // the query tile is free once the item's last Q K^T is done
                     if (j == n_kt - 1) umma_commit(&bar[kQEmpty]);
                     issued = true;
@@ -376,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quarter = warp & 3;         // TMEM lanes 32*quarter .. +31
         const int r = quarter * 32 + lane;    // the row of the tile
         const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
-        const uint32_t tS = tmem + lanes, tO = tmem + lanes + kBN;
+        const uint32_t tS = tmem + lanes, tO = tmem + lanes + kBN, tP = tmem + lanes + 2 * kBN;
         int64_t g = 0;
         bool stop = false;
         for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
@@ -437,23 +477,35 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
                     pk[i / 2] = *reinterpret_cast<uint32_t *>(&h);
                 }
-                if (j > 0) {
-                    // O holds the earlier tiles' sum (and P is free) once PV(j-1) is done
-                    if (!__all_sync(0xffffffffu,
-                                    wait_bar(&bar[kOFull], (uint32_t)((g - 1) & 1), abort, err))) {
+                // P of this tile goes to TMEM buffer g & 1, free once the P V
+                // of tile g - 2 is done
+                const int pb = (int)(g & 1);
+                if (g >= 2 && !__all_sync(0xffffffffu,
+                                          wait_bar(&bar[kPFree + pb], (uint32_t)(((g >> 1) - 1) & 1),
+                                                   abort, err))) {
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                tmem_st64(tP + pb * (kBN / 2), pk);
+                if (j > 0 && __any_sync(0xffffffffu, bump)) {
+                    // rescale O, which holds the earlier tiles' sum once the P V of
+                    // tile g - 1 is done
+                    const int qb = (int)((g - 1) & 1);
+                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kPFree + qb],
+                                                          (uint32_t)(((g - 1) >> 1) & 1), abort,
+                                                          err))) {
                         stop = true;
                         break;
                     }
                     tc_fence_after();
-                    if (__any_sync(0xffffffffu, bump)) {
-                        uint32_t o[128];
-                        tmem_ld128(tO, o);
+                    uint32_t o[128];
+                    tmem_ld128(tO, o);
 #pragma unroll
-                        for (int i = 0; i < 128; i++)
-                            o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
-                        tmem_st128(tO, o);
-                        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-                    }
+                    for (int i = 0; i < 128; i++)
+                        o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
+                    tmem_st128(tO, o);
+                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 }
                 l = l * corr + rowsum;
                 m = mu;
@@ -473,22 +525,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                             *reinterpret_cast<uint4 *>(row + kHalf + x * 16) = make_uint4(0, 0, 0, 0);
                         }
                     }
+                    fence_proxy_async_shared();  // the MMA reads these rows
                 }
-                // P row r in the 128-byte swizzled K-major layout of the MMA's A operand
-#pragma unroll
-                for (int c16 = 0; c16 < 16; c16++) {
-                    unsigned char *dst =
-                        sP + (c16 >> 3) * kHalf + r * 128 + (((c16 & 7) ^ (r & 7)) * 16);
-                    *reinterpret_cast<uint4 *>(dst) =
-                        make_uint4(pk[4 * c16], pk[4 * c16 + 1], pk[4 * c16 + 2], pk[4 * c16 + 3]);
-                }
-                fence_proxy_async_shared();
                 tc_fence_before();
-                mbar_arrive(&bar[kPFull]);
+                mbar_arrive(&bar[kPFull + pb]);
             }
             if (stop) break;
-            // epilogue: O / l once the last PV is done
-            if (!__all_sync(0xffffffffu, wait_bar(&bar[kOFull], (uint32_t)((g - 1) & 1), abort, err)))
+            // epilogue: O / l once the last P V is done
+            if (!__all_sync(0xffffffffu, wait_bar(&bar[kPFree + ((g - 1) & 1)],
+                                                  (uint32_t)(((g - 1) >> 1) & 1), abort, err)))
                 break;
             tc_fence_after();
             const float inv = 1.f / l;
