@@ -138,6 +138,46 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full,
                               speechkv_dtype dtype, cudaStream_t stream);
 
 /*
+ * speechkv_pool_hidden -- the HS-compression variant (Sec. IV-A): the
+ * pooling of Eq. (pool) applied once, at layer l0, to the whole hidden
+ * state instead of to each layer's keys and values, so that every later
+ * layer (queries included) runs on the shorter sequence.
+ *
+ * For every request b: text rows are copied bit-exactly; speech window i
+ * (frames i*w .. min((i+1)*w, T) - 1 of the speech span) becomes one row
+ * with logits z_j = gate . h_j over the whole hidden vector, weights
+ * alpha = softmax(z) over the window and h^ = sum alpha_j h_j, rounded once
+ * to the storage type.  Output rows [P; pooled n; N] of request b start at
+ * row out_off[b]; len[b] = P[b] + ceil(T[b] / w) + N[b].  w = 1 copies.
+ *
+ * h_full     dev, [full_rows][d_model] token-major hidden states; request b's
+ *            rows are [full_off[b], full_off[b+1]) and must be P+T+N rows.
+ * full_off   dev int64 [B+1].
+ * P, T, N    dev int32 [B], as for speechkv_pool.
+ * gate       dev fp32 [d_model]: the gate vector u of g(h) = u . h.
+ * h_out      dev, [out_rows][d_model]; out_off dev int64 [B+1] gives each
+ *            request's rows (capacity out_off[b+1] - out_off[b]).
+ * len        dev int32 [B], written.
+ * full_rows, out_rows  host: rows of h_full and h_out.
+ * Supported: SPEECHKV_F32 or SPEECHKV_BF16 with d_model * element size a
+ * multiple of 16 bytes and at most 16 KB (SPEECHKV_ERR_UNSUPPORTED
+ * otherwise).  On the device, a request whose rows do not match P+T+N or
+ * lie outside full_rows / out_rows sets SPEECHKV_ERR_INVALID_ARG; one whose
+ * pooled rows exceed its capacity sets SPEECHKV_ERR_CAPACITY (rows beyond
+ * the capacity are not written and len is clamped).
+ */
+speechkv_status speechkv_pool_hidden(const void *h_full,
+                                     const int64_t *full_off,
+                                     const int32_t *P, const int32_t *T,
+                                     const int32_t *N, const float *gate,
+                                     void *h_out, const int64_t *out_off,
+                                     int32_t *len, int32_t B,
+                                     int64_t full_rows, int64_t out_rows,
+                                     int32_t d_model, int32_t w,
+                                     speechkv_dtype dtype,
+                                     cudaStream_t stream);
+
+/*
  * speechkv_prefill_attn -- Eq. (attn) at prefill (Sec. III-B): every
  * full-resolution prompt query attends over the compressed cache rows that
  * precede it.

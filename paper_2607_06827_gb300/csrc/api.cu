@@ -237,6 +237,48 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full, const int6
                                                                        : SPEECHKV_ERR_CUDA;
 }
 
+speechkv_status speechkv_pool_hidden(const void *h_full, const int64_t *full_off,
+                                     const int32_t *P, const int32_t *T, const int32_t *N,
+                                     const float *gate, void *h_out, const int64_t *out_off,
+                                     int32_t *len, int32_t B, int64_t full_rows,
+                                     int64_t out_rows, int32_t d_model, int32_t w,
+                                     speechkv_dtype dtype, cudaStream_t stream) {
+    if (B < 0 || full_rows < 0 || out_rows < 0 || d_model < 1 || w < 1 || !valid_dtype(dtype))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!speechkv::pool_hidden_supported(dtype, d_model)) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!full_off || !P || !T || !N || !gate || !h_out || !out_off || !len ||
+        (full_rows > 0 && !h_full))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(h_full, 16) || !aligned(h_out, 16) || !aligned(full_off, 8) ||
+        !aligned(out_off, 8) || !aligned(P, 4) || !aligned(T, 4) || !aligned(N, 4) ||
+        !aligned(len, 4) || !aligned(gate, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::PoolHiddenArgs a;
+    a.h_full = h_full;
+    a.full_off = full_off;
+    a.P = P;
+    a.T = T;
+    a.N = N;
+    a.gate = gate;
+    a.h_out = h_out;
+    a.out_off = out_off;
+    a.len = len;
+    a.B = B;
+    a.full_rows = full_rows;
+    a.out_rows = out_rows;
+    a.d_model = d_model;
+    a.w = w;
+    a.dtype = dtype;
+    a.err = s->err;
+    return speechkv::launch_pool_hidden(a, s->num_sms, stream) == cudaSuccess
+               ? SPEECHKV_OK
+               : SPEECHKV_ERR_CUDA;
+}
+
 speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64_t q_rows,
                                       const int32_t *P, const int32_t *T, const int32_t *N,
                                       const void *k_cache, const void *v_cache,

@@ -25,6 +25,24 @@ struct PoolArgs {
 };
 cudaError_t launch_pool(const PoolArgs &a, int num_sms, cudaStream_t stream);
 
+struct PoolHiddenArgs {
+    const void *h_full;  // [full_rows][d_model]
+    const int64_t *full_off;
+    const int32_t *P, *T, *N;
+    const float *gate;   // [d_model]
+    void *h_out;         // [out_rows][d_model]
+    const int64_t *out_off;
+    int32_t *len;
+    int32_t B;
+    int64_t full_rows, out_rows;
+    int32_t d_model, w;
+    speechkv_dtype dtype;
+    int *err;
+};
+// Whether (dtype, d_model) is supported by the hidden-state pooling kernel.
+bool pool_hidden_supported(speechkv_dtype dtype, int d_model);
+cudaError_t launch_pool_hidden(const PoolHiddenArgs &a, int num_sms, cudaStream_t stream);
+
 struct AppendArgs {
     const void *k_new, *v_new;
     void *k_cache, *v_cache;

@@ -264,6 +264,176 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Hidden-state pooling (the HS-compression variant): the same operator on
+// whole hidden vectors, h^_i = sum_j alpha_j h_j with alpha = softmax over the
+// window of gate . h_j.  A CTA of 256 threads handles one output row at a
+// time; each thread owns up to kHsVpt 16-byte vectors of the row, the logits
+// of up to kPoolFrames frames are reduced across the CTA together.
+// ---------------------------------------------------------------------------
+constexpr int kHsThreads = 256;
+constexpr int kHsVptMax = 4;  // 16-byte vectors per thread: d_model * sizeof(T) <= 16 KB
+
+template <typename T, int kHsVpt>
+__global__ void __launch_bounds__(kHsThreads)
+    pool_hidden_kernel(const T *__restrict__ hf, const int64_t *__restrict__ full_off,
+                       const int32_t *__restrict__ Pa, const int32_t *__restrict__ Ta,
+                       const int32_t *__restrict__ Na, const float *__restrict__ gate,
+                       T *__restrict__ ho, const int64_t *__restrict__ out_off,
+                       int32_t *__restrict__ len, int64_t full_rows, int64_t out_rows, int VR,
+                       int w, int *__restrict__ err) {
+    constexpr int EPV = 16 / (int)sizeof(T), NP = EPV / 2;
+    constexpr int kWarps = kHsThreads / 32;
+    __shared__ float red[kPoolFrames][kWarps];
+    const int b = blockIdx.y;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+    const int64_t row0 = full_off[b], S = full_off[b + 1] - row0;
+    const int64_t base = out_off[b], cap = out_off[b + 1] - base;
+    const int64_t Pb = Pa[b], Tb = Ta[b], Nb = Na[b];
+    const int64_t n = (Tb + w - 1) / w;
+    const int64_t L = Pb + n + Nb;
+    const bool bad = Pb < 0 || Tb < 0 || Nb < 0 || S != Pb + Tb + Nb || cap < 0 || row0 < 0 ||
+                     full_off[b + 1] > full_rows || base < 0 || out_off[b + 1] > out_rows;
+    if (blockIdx.x == 0 && tid == 0) {
+        if (bad)
+            report_error(err, SPEECHKV_ERR_INVALID_ARG);
+        else if (L > cap)
+            report_error(err, SPEECHKV_ERR_CAPACITY);
+        len[b] = (int32_t)(bad ? 0 : (L < cap ? L : cap));
+    }
+    if (bad) return;
+    const int64_t rows_out = L < cap ? L : cap;
+    const uint4 *src = reinterpret_cast<const uint4 *>(hf) + row0 * VR;
+    uint4 *dst = reinterpret_cast<uint4 *>(ho) + base * VR;
+
+    // the thread's slice of the gate, scaled by log2(e) (softmax in base 2)
+    constexpr float kLog2e = 1.4426950408889634f;
+    float2 u[kHsVpt][NP];
+#pragma unroll
+    for (int x = 0; x < kHsVpt; x++) {
+        const int v = tid + x * kHsThreads;
+#pragma unroll
+        for (int k = 0; k < NP; k++) {
+            u[x][k] = v < VR ? make_float2(gate[v * EPV + 2 * k] * kLog2e,
+                                           gate[v * EPV + 2 * k + 1] * kLog2e)
+                             : make_float2(0.f, 0.f);
+        }
+    }
+
+    for (int64_t t = blockIdx.x; t < rows_out; t += gridDim.x) {
+        if (t < Pb || t >= Pb + n || w == 1) {
+            // text row (or no pooling): bit-exact copy
+            const int64_t s = (t < Pb || w == 1) ? t : t - n + Tb;
+#pragma unroll
+            for (int x = 0; x < kHsVpt; x++) {
+                const int v = tid + x * kHsThreads;
+                if (v < VR) dst[t * VR + v] = __ldcs(src + s * VR + v);
+            }
+            continue;
+        }
+        const int64_t j0 = Pb + (t - Pb) * w;
+        const int64_t j1 = (j0 + w < Pb + Tb) ? j0 + w : Pb + Tb;
+        float m = -INFINITY, l = 0.f;
+        float2 acc[kHsVpt][NP];
+#pragma unroll
+        for (int x = 0; x < kHsVpt; x++)
+#pragma unroll
+            for (int k = 0; k < NP; k++) acc[x][k] = make_float2(0.f, 0.f);
+        for (int64_t j = j0; j < j1; j += kPoolFrames) {
+            const int nf = j1 - j < kPoolFrames ? (int)(j1 - j) : kPoolFrames;
+            uint4 raw[kPoolFrames][kHsVpt];
+            float z[kPoolFrames];
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++) {
+                float2 a2 = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int x = 0; x < kHsVpt; x++) {
+                    const int v = tid + x * kHsThreads;
+                    raw[f][x] = (f < nf && v < VR) ? __ldcs(src + (j + f) * VR + v)
+                                                   : make_uint4(0u, 0u, 0u, 0u);
+                    float2 e[NP];
+                    widen2<T>(raw[f][x], e);
+#pragma unroll
+                    for (int k = 0; k < NP; k++) a2 = ffma2(u[x][k], e[k], a2);
+                }
+                z[f] = warp_sum(a2.x + a2.y);
+            }
+            // CTA-wide sums of the frames' logits (fixed order: deterministic)
+            if (lane == 0)
+#pragma unroll
+                for (int f = 0; f < kPoolFrames; f++) red[f][warp] = z[f];
+            __syncthreads();
+            float mb = m;
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++) {
+                float zz = 0.f;
+#pragma unroll
+                for (int x = 0; x < kWarps; x++) zz += red[f][x];
+                z[f] = zz;
+                if (f < nf) mb = fmaxf(mb, zz);
+            }
+            __syncthreads();  // red[] is rewritten by the next frames
+            const float corr = fast_exp2(m - mb);  // 0 on the first frames
+            l *= corr;
+#pragma unroll
+            for (int x = 0; x < kHsVpt; x++)
+#pragma unroll
+                for (int k = 0; k < NP; k++) acc[x][k] = fmul2(acc[x][k], make_float2(corr, corr));
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++) {
+                if (f >= nf) break;
+                const float p = fast_exp2(z[f] - mb);
+                l += p;
+#pragma unroll
+                for (int x = 0; x < kHsVpt; x++) {
+                    float2 e[NP];
+                    widen2_prmt<T>(raw[f][x], e);
+#pragma unroll
+                    for (int k = 0; k < NP; k++) acc[x][k] = ffma2(make_float2(p, p), e[k], acc[x][k]);
+                }
+            }
+            m = mb;
+        }
+        const float inv = 1.f / l;
+#pragma unroll
+        for (int x = 0; x < kHsVpt; x++) {
+            const int v = tid + x * kHsThreads;
+            if (v >= VR) continue;
+            float o[EPV];
+#pragma unroll
+            for (int k = 0; k < NP; k++) {
+                o[2 * k] = acc[x][k].x * inv;
+                o[2 * k + 1] = acc[x][k].y * inv;
+            }
+            store_vec<T, EPV>(reinterpret_cast<T *>(dst + t * VR + v), o);
+        }
+    }
+}
+
+template <typename T, int VPT>
+cudaError_t launch_pool_hidden_vpt(const PoolHiddenArgs &a, const dim3 &grid, int VR,
+                                   cudaStream_t stream) {
+    pool_hidden_kernel<T, VPT><<<grid, kHsThreads, 0, stream>>>(
+        static_cast<const T *>(a.h_full), a.full_off, a.P, a.T, a.N, a.gate,
+        static_cast<T *>(a.h_out), a.out_off, a.len, a.full_rows, a.out_rows, VR, a.w, a.err);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_pool_hidden_instance(const PoolHiddenArgs &a, int num_sms,
+                                        cudaStream_t stream) {
+    int64_t x = ((int64_t)4 * num_sms + a.B - 1) / a.B;
+    if (x < 1) x = 1;
+    if (x > 65535) x = 65535;
+    const dim3 grid((unsigned)x, (unsigned)a.B);
+    const int VR = (int)((int64_t)a.d_model * (int64_t)sizeof(T) / 16);
+    const int vpt = (VR + kHsThreads - 1) / kHsThreads;
+    if (vpt <= 1) return launch_pool_hidden_vpt<T, 1>(a, grid, VR, stream);
+    if (vpt <= 2) return launch_pool_hidden_vpt<T, 2>(a, grid, VR, stream);
+    return launch_pool_hidden_vpt<T, kHsVptMax>(a, grid, VR, stream);
+}
+
 template <typename T, int D>
 cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t stream) {
     // enough CTAs over the whole batch to fill every SM once, at least one
@@ -288,6 +458,17 @@ cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t st
 }
 
 }  // namespace
+
+bool pool_hidden_supported(speechkv_dtype dtype, int d_model) {
+    const int es = dtype == SPEECHKV_F32 ? 4 : 2;
+    return d_model > 0 && (d_model * es) % 16 == 0 && d_model * es <= kHsVptMax * kHsThreads * 16;
+}
+
+cudaError_t launch_pool_hidden(const PoolHiddenArgs &a, int num_sms, cudaStream_t stream) {
+    if (a.B > 65535) return cudaErrorInvalidValue;  // grid.y limit
+    if (a.dtype == SPEECHKV_F32) return launch_pool_hidden_instance<float>(a, num_sms, stream);
+    return launch_pool_hidden_instance<__nv_bfloat16>(a, num_sms, stream);
+}
 
 cudaError_t launch_pool(const PoolArgs &a, int num_sms, cudaStream_t stream) {
     if (a.B > 65535) return cudaErrorInvalidValue;  // grid.y limit

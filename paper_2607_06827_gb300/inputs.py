@@ -127,6 +127,7 @@ def qwen_ragged(B: int = 128, w: int = 4, seed: int = 1005) -> Workload:
 TAG_PREFILL_K, TAG_PREFILL_V, TAG_GATE = 1, 2, 3
 TAG_Q, TAG_KNEW, TAG_VNEW, TAG_GEN_K, TAG_GEN_V = 4, 5, 6, 7, 8
 TAG_PREFILL_Q = 9
+TAG_HIDDEN, TAG_HIDDEN_GATE = 10, 11
 
 
 def rng_for(seed: int, *key: int) -> np.random.Generator:
@@ -162,6 +163,17 @@ def prefill_q(wl: Workload, layer: int, b: int):
     S = wl.P[b] + wl.T[b] + wl.N[b]
     q = normal_f32(wl.seed, (TAG_PREFILL_Q, layer, b), (S, wl.H_q, wl.d))
     return to_storage(q, wl.dtype)
+
+
+def hidden_states(wl: Workload, b: int, d_model: int):
+    """Hidden states of request b's prompt at the pooling layer: [P+T+N, d_model]."""
+    S = wl.P[b] + wl.T[b] + wl.N[b]
+    return to_storage(normal_f32(wl.seed, (TAG_HIDDEN, b), (S, d_model)), wl.dtype)
+
+
+def hidden_gate(wl: Workload, d_model: int, scale: float = 1.0) -> np.ndarray:
+    """Gate vector u ~ N(0, scale^2 / d_model) over the hidden state, fp32 [d_model]."""
+    return normal_f32(wl.seed, (TAG_HIDDEN_GATE,), (d_model,), std=scale / np.sqrt(d_model))
 
 
 def generated_kv(wl: Workload, layer: int, b: int):

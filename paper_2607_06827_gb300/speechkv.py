@@ -46,6 +46,8 @@ SIGNATURES = {
                                                     _I32, _I32, _I32, _I32, _I32, _I32,
                                                     _I32, _I32, ctypes.c_int,
                                                     ctypes.c_uint32, _P]),
+    "speechkv_pool_hidden": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _I32, _I64,
+                                            _I64, _I32, _I32, ctypes.c_int, _P]),
     "speechkv_prefill_attn": (ctypes.c_int, [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _I64, _P, _F,
                                              _I32, _I32, _I32, _I32, _I32, _I32, _I32,
                                              ctypes.c_int, _P]),
@@ -195,6 +197,19 @@ def decode_step_noalloc(q, k_new, v_new, k_cache, v_cache, cache_off, length, ou
         _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas,
         _dtype_code(q), flags, _stream(stream)),
         "speechkv_decode_step_noalloc")
+
+
+def pool_hidden(h_full, full_off, P, T, N, gate, h_out, out_off, length, w: int, stream=None):
+    """speechkv_pool_hidden: h_full [full_rows, d_model] -> h_out
+    [out_rows, d_model] (HS-compression variant); full_off/out_off int64
+    [B+1]; P/T/N/length int32 [B]; gate fp32 [d_model]."""
+    B = length.numel()
+    full_rows, d_model = h_full.shape
+    _check(load().speechkv_pool_hidden(
+        _ptr(h_full), _ptr(full_off), _ptr(P), _ptr(T), _ptr(N), _ptr(gate), _ptr(h_out),
+        _ptr(out_off), _ptr(length), B, full_rows, h_out.shape[0], d_model, w,
+        _dtype_code(h_full), _stream(stream)),
+        "speechkv_pool_hidden")
 
 
 def prefill_attn(q, q_off, P, T, N, k_cache, v_cache, cache_off, out, w: int, layer: int,

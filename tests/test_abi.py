@@ -79,6 +79,14 @@ def test_host_argument_checks_without_gpu():
     assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 128, 0, 0, 0, sk.BF16, z) == sk.ERR_INVALID_ARG
     assert lib.speechkv_pool(*([z] * 11), 1, 10, 8, 80, 4, 0, 0, sk.BF16, z) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_pool(*([z] * 11), 0, 0, 8, 128, 4, 0, 0, sk.BF16, z) == sk.OK
+    # hidden-state pooling: d_model * element size a multiple of 16 bytes, <= 16 KB
+    ph = lambda B, d_model, w, dt: (*([z] * 9), B, 10, 10, d_model, w, dt, z)  # noqa: E731
+    assert lib.speechkv_pool_hidden(*ph(1, 2048, 0, sk.BF16)) == sk.ERR_INVALID_ARG
+    assert lib.speechkv_pool_hidden(*ph(1, 2044, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_pool_hidden(*ph(1, 16384, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_pool_hidden(*ph(0, 2048, 4, sk.BF16)) == sk.OK
+    assert lib.speechkv_pool_hidden(*ph(1, 2048, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
+    assert lib.speechkv_pool_hidden(*ph(1, 4096, 4, sk.F32)) == sk.ERR_INVALID_ARG   # NULLs
     # prefill attention: bf16 and d = 128 only; 32-bit tensor-copy coordinates
     pf = lambda B, q_rows, cache_rows, H_q, H_kv, d, w, dt: (  # noqa: E731
         z, z, q_rows, z, z, z, z, z, z, cache_rows, z, 0.0, B, H_q, H_kv, d, w, 0, 0, dt, z)

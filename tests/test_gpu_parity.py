@@ -5,6 +5,7 @@ Eq. (attn); Sec. III-C for the prefill-once / append-per-step cache).
 Tolerances: fp32 max-abs 1e-5; bf16 max-abs 2e-2 and mean-abs 2e-3 on
 unit-variance inputs; lengths, offsets and copied rows bit-exact.
 """
+import dataclasses
 import math
 
 import numpy as np
@@ -332,6 +333,16 @@ def test_end_to_end_qwen_single(sk, oracle):
 def test_end_to_end_ragged_small(sk, oracle):
     wl = inputs.qwen_ragged(B=6)
     _run_steps(sk, oracle, wl, layers=[wl.l0], steps=3)
+
+
+def test_per_layer_windows(sk, oracle):
+    """Compression ratios that differ across layers (the paper leaves adaptive
+    ratios to future work): the window is an argument of every call, so each
+    layer's cache may be pooled with its own w.  Layers 7 (before l0), 8, 9, 10
+    with w = 4 (unused: full resolution), 2, 4, 8; fused decode steps."""
+    base = inputs.qwen_single()
+    for layer, w in ((base.l0 - 1, 4), (base.l0, 2), (base.l0 + 1, 4), (base.l0 + 2, 8)):
+        _run_steps(sk, oracle, dataclasses.replace(base, w=w), layers=[layer], steps=3, fused=True)
 
 
 # --------------------------------------------------------------------------
