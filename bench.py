@@ -533,10 +533,58 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
     peak, kind = measured_bf16_peak()
     for r in res.values():
         r["frac"] = round(r["tflops"] / peak, 4)
+    res["hs_pool"] = measure_hs_pool(wl, clocks, repeats, warmup)
     res.update({"bound": "tensor", "peak": peak, "peak_kind": kind, "unit": "TFLOP/s",
                 "kernel": "prefill_attn_kernel (tcgen05, bf16, d=128): speechkv_prefill_attn",
                 "workload": f"whole prompt of the batch ({S} query rows x {wl.H_q} heads)"})
     return res
+
+
+def measure_hs_pool(wl, clocks, repeats: int = 5, warmup: int = 2, d_model: int = 2048):
+    """speechkv_pool_hidden (the HS-compression variant) on the whole prompt
+    of the batch: Qwen3-1.7B hidden states (d_model 2048, bf16) pooled with w.
+    Algorithmic bytes = rows read + rows written; GB/s against the measured
+    HBM peak."""
+    import numpy as np
+    import torch
+    from paper_2607_06827_gb300 import inputs, speechkv as sk
+    rows_in = wl.full_rows()
+    rows_out = [sk.compressed_len(p, t, n, 0, wl.w, 0, 0) for p, t, n in zip(wl.P, wl.T, wl.N)]
+    off = lambda r: torch.from_numpy(np.concatenate([[0], np.cumsum(r)]).astype(np.int64)).cuda()  # noqa: E731
+    full_off, out_off = off(rows_in), off(rows_out)
+    t32 = lambda x: torch.tensor(x, dtype=torch.int32, device="cuda")  # noqa: E731
+    P, T, N = t32(wl.P), t32(wl.T), t32(wl.N)
+    h = inputs.device_normal((sum(rows_in), d_model), torch.bfloat16, "cuda", wl.seed, 43)
+    gate = inputs.device_normal((d_model,), torch.float32, "cuda", wl.seed, 44) / math.sqrt(d_model)
+    out = torch.empty((sum(rows_out), d_model), dtype=torch.bfloat16, device="cuda")
+    ln = torch.zeros(wl.B, dtype=torch.int32, device="cuda")
+
+    def launch():
+        sk.pool_hidden(h, full_off, P, T, N, gate, out, out_off, ln, wl.w)
+    for _ in range(warmup):
+        launch()
+    torch.cuda.synchronize()
+    times = []
+    t0 = time.time()
+    for _ in range(repeats):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        launch()
+        e1.record()
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    clocks and clocks.mark(t0, time.time())
+    status = sk.check_device_error()
+    assert status == sk.OK, sk.status_string(status)
+    ms = sorted(times)[len(times) // 2]
+    nbytes = (sum(rows_in) + sum(rows_out)) * d_model * 2
+    peak, kind = measured_peak()
+    gbs = nbytes / (ms * 1e-3) / 1e9
+    del h, out
+    torch.cuda.empty_cache()
+    return {"us": round(ms * 1e3, 1), "bytes": nbytes, "gbs": round(gbs, 1),
+            "frac": round(gbs / peak, 4), "peak": peak, "peak_kind": kind, "d_model": d_model,
+            "kernel": "pool_hidden_kernel: speechkv_pool_hidden (HS-compression variant)"}
 
 
 # ---------------------------------------------------------------------------
