@@ -361,6 +361,56 @@ speechkv_status speechkv_decode_step_noalloc(
     uint32_t flags, cudaStream_t stream);
 
 /*
+ * Paged caches -- the block-table layout of the paper's serving system (a
+ * vLLM-style paged KV cache, Sec. V-D); the paper has no other use for it.
+ * A layer's keys and values live in fixed-size pages
+ *     k_pages, v_pages   dev, [num_blocks][H_kv][block_size][d]
+ * and request b's logical rows t are found through its block-table row:
+ *     row t -> page block_table[b * max_blocks + t / block_size],
+ *              slot t % block_size of that page (every KV head's slot).
+ * block_table  dev int32 [B][max_blocks]; an entry is a page index in
+ *              [0, num_blocks) for every row the call reads or writes
+ *              (others may hold anything, e.g. -1).
+ * block_size   a power of two; each request's capacity is
+ *              max_blocks * block_size rows (at most 2^31 - 1).
+ * num_blocks   host: pages in k_pages / v_pages (bounds the table entries).
+ * The other arguments, the results and the errors are those of the
+ * contiguous entry point of the same name (the rows and their order are the
+ * same; only where they live differs).  A table entry outside [0, num_blocks)
+ * where a row is needed sets SPEECHKV_ERR_INVALID_ARG on the device; that
+ * row is neither written nor used (its contents in the result are
+ * unspecified).
+ */
+speechkv_status speechkv_pool_paged(const void *k_full, const void *v_full,
+                                    const int64_t *full_off, const int32_t *P,
+                                    const int32_t *T, const int32_t *N,
+                                    const float *gate, void *k_pages,
+                                    void *v_pages, const int32_t *block_table,
+                                    int32_t max_blocks, int32_t block_size,
+                                    int64_t num_blocks, int32_t *len,
+                                    int32_t B, int64_t full_rows, int32_t H_kv,
+                                    int32_t d, int32_t w, int32_t layer,
+                                    int32_t l0, speechkv_dtype dtype,
+                                    cudaStream_t stream);
+speechkv_status speechkv_append_paged(const void *k_new, const void *v_new,
+                                      void *k_pages, void *v_pages,
+                                      const int32_t *block_table,
+                                      int32_t max_blocks, int32_t block_size,
+                                      int64_t num_blocks, int32_t *len,
+                                      int32_t B, int32_t H_kv, int32_t d,
+                                      int32_t w, int32_t layer, int32_t l0,
+                                      speechkv_dtype dtype,
+                                      cudaStream_t stream);
+speechkv_status speechkv_decode_step_paged(
+    const void *q, const void *k_new, const void *v_new, void *k_pages,
+    void *v_pages, const int32_t *block_table, int32_t max_blocks,
+    int32_t block_size, int64_t num_blocks, int32_t *len, void *out,
+    float scale, int32_t B, int32_t H_q, int32_t H_kv, int32_t d, int32_t w,
+    int32_t layer, int32_t l0, int32_t grid_ctas, void *workspace,
+    size_t workspace_bytes, speechkv_dtype dtype, uint32_t flags,
+    cudaStream_t stream);
+
+/*
  * Synchronises `stream`, then reads and clears the current device's error
  * word.  Returns SPEECHKV_OK when no kernel reported an error since the last
  * check, else the first error reported (CAPACITY, INVALID_ARG or TIMEOUT),

@@ -117,7 +117,7 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
                               int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
                               int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
                               speechkv_dtype dtype, uint32_t flags, cudaStream_t stream,
-                              bool append) {
+                              bool append, const speechkv::CacheMap &map = {}) {
     if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
         grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale) ||
         (flags & ~SPEECHKV_OVERLAP_PRIOR))
@@ -125,7 +125,7 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
     if (!speechkv::decode_supported(dtype, d, H_q / H_kv)) return SPEECHKV_ERR_UNSUPPORTED;
     if (B > SPEECHKV_MAX_BATCH) return SPEECHKV_ERR_UNSUPPORTED;
     if (B == 0) return SPEECHKV_OK;
-    if (!q || !k_cache || !v_cache || !cache_off || !len || !out ||
+    if (!q || !k_cache || !v_cache || (!cache_off && !map.table) || !len || !out ||
         (append && (!k_new || !v_new)))
         return SPEECHKV_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
@@ -164,9 +164,39 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
                                            counters_bytes(B, H_kv));
     a.err = s->err;
     a.overlap = (flags & SPEECHKV_OVERLAP_PRIOR) != 0;
+    a.map = map;
     return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
                                                                    : SPEECHKV_ERR_CUDA;
 }
+
+// Host checks of a block table's description (the table itself is read on
+// the device, where a bad entry is reported, not followed).
+speechkv_status make_map(const int32_t *block_table, int32_t max_blocks, int32_t block_size,
+                         int64_t num_blocks, speechkv::CacheMap *m) {
+    if (!block_table || !aligned(block_table, 4) || max_blocks < 1 || num_blocks < 1 ||
+        block_size < 1 || (block_size & (block_size - 1)) != 0 || block_size > (1 << 20))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if ((int64_t)max_blocks * block_size > INT32_MAX) return SPEECHKV_ERR_UNSUPPORTED;
+    int lg = 0;
+    while ((1 << lg) < block_size) lg++;
+    m->table = block_table;
+    m->max_blocks = max_blocks;
+    m->bs_log2 = lg;
+    m->num_blocks = num_blocks;
+    return SPEECHKV_OK;
+}
+
+speechkv_status pool_impl(const void *k_full, const void *v_full, const int64_t *full_off,
+                          const int32_t *P, const int32_t *T, const int32_t *N, const float *gate,
+                          void *k_cache, void *v_cache, const int64_t *cache_off, int32_t *len,
+                          int32_t B, int64_t full_rows, int32_t H_kv, int32_t d, int32_t w,
+                          int32_t layer, int32_t l0, speechkv_dtype dtype, cudaStream_t stream,
+                          const speechkv::CacheMap &map);
+speechkv_status append_impl(const void *k_new, const void *v_new, void *k_cache, void *v_cache,
+                            const int64_t *cache_off, int32_t *len, int32_t B, int32_t H_kv,
+                            int32_t d, int32_t w, int32_t layer, int32_t l0,
+                            speechkv_dtype dtype, cudaStream_t stream,
+                            const speechkv::CacheMap &map);
 
 }  // namespace
 
@@ -199,42 +229,98 @@ speechkv_status speechkv_pool(const void *k_full, const void *v_full, const int6
                               int64_t full_rows, int32_t H_kv, int32_t d, int32_t w,
                               int32_t layer, int32_t l0, speechkv_dtype dtype,
                               cudaStream_t stream) {
-    if (B < 0 || full_rows < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
+    return pool_impl(k_full, v_full, full_off, P, T, N, gate, k_cache, v_cache, cache_off, len, B,
+                     full_rows, H_kv, d, w, layer, l0, dtype, stream, {});
+}
+
+speechkv_status speechkv_pool_paged(const void *k_full, const void *v_full,
+                                    const int64_t *full_off, const int32_t *P, const int32_t *T,
+                                    const int32_t *N, const float *gate, void *k_pages,
+                                    void *v_pages, const int32_t *block_table,
+                                    int32_t max_blocks, int32_t block_size, int64_t num_blocks,
+                                    int32_t *len, int32_t B, int64_t full_rows, int32_t H_kv,
+                                    int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                    speechkv_dtype dtype, cudaStream_t stream) {
+    speechkv::CacheMap m;
     if (B == 0) return SPEECHKV_OK;
-    if (!full_off || !P || !T || !N || !gate || !k_cache || !v_cache || !cache_off || !len ||
-        (full_rows > 0 && (!k_full || !v_full)))
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (!aligned(k_full, 16) || !aligned(v_full, 16) || !aligned(k_cache, 16) ||
-        !aligned(v_cache, 16) || !aligned(full_off, 8) || !aligned(cache_off, 8) ||
-        !aligned(P, 4) || !aligned(T, 4) || !aligned(N, 4) || !aligned(len, 4) ||
-        !aligned(gate, 16))
-        return SPEECHKV_ERR_INVALID_ARG;
+    const speechkv_status st = make_map(block_table, max_blocks, block_size, num_blocks, &m);
+    if (st != SPEECHKV_OK) return st;
+    return pool_impl(k_full, v_full, full_off, P, T, N, gate, k_pages, v_pages, nullptr, len, B,
+                     full_rows, H_kv, d, w, layer, l0, dtype, stream, m);
+}
+
+speechkv_status speechkv_append(const void *k_new, const void *v_new, void *k_cache,
+                                void *v_cache, const int64_t *cache_off, int32_t *len,
+                                int32_t B, int32_t H_kv, int32_t d, int32_t w, int32_t layer,
+                                int32_t l0, speechkv_dtype dtype, cudaStream_t stream) {
+    return append_impl(k_new, v_new, k_cache, v_cache, cache_off, len, B, H_kv, d, w, layer, l0,
+                       dtype, stream, {});
+}
+
+speechkv_status speechkv_append_paged(const void *k_new, const void *v_new, void *k_pages,
+                                      void *v_pages, const int32_t *block_table,
+                                      int32_t max_blocks, int32_t block_size,
+                                      int64_t num_blocks, int32_t *len, int32_t B,
+                                      int32_t H_kv, int32_t d, int32_t w, int32_t layer,
+                                      int32_t l0, speechkv_dtype dtype, cudaStream_t stream) {
+    speechkv::CacheMap m;
+    if (B == 0) return SPEECHKV_OK;
+    const speechkv_status st = make_map(block_table, max_blocks, block_size, num_blocks, &m);
+    if (st != SPEECHKV_OK) return st;
+    return append_impl(k_new, v_new, k_pages, v_pages, nullptr, len, B, H_kv, d, w, layer, l0,
+                       dtype, stream, m);
+}
+
+
+size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv, int32_t d,
+                                      int32_t grid_ctas) {
+    if (B < 0 || H_kv < 1 || H_q < 1 || H_q % H_kv != 0 || grid_ctas < 0) return 0;
+    if (!speechkv::decode_supported(SPEECHKV_BF16, d, H_q / H_kv)) return 0;
+    int grid = grid_ctas;
+    if (grid == 0) {
+        DeviceState *s = nullptr;
+        if (device_state(&s) != SPEECHKV_OK) return 0;
+        grid = s->num_sms * kAutoCtasPerSmMax;
+    }
+    return workspace_bytes(B, H_q, H_kv, d, grid);
+}
+
+speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const void *v_cache,
+                                     const int64_t *cache_off, const int32_t *len, void *out,
+                                     float scale, int32_t B, int32_t H_q, int32_t H_kv,
+                                     int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
+    // the caches and len are only read on this path
+    return decode_common(q, nullptr, nullptr, const_cast<void *>(k_cache),
+                         const_cast<void *>(v_cache), cache_off, const_cast<int32_t *>(len), out,
+                         scale, B, H_q, H_kv, d, w, layer, l0, grid_ctas, workspace,
+                         workspace_bytes_in, dtype, flags, stream, false);
+}
+
+speechkv_status speechkv_decode_step(const void *q, const void *k_new, const void *v_new,
+                                     void *k_cache, void *v_cache, const int64_t *cache_off,
+                                     int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+                                     int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
+    return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
+                         H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
+                         flags, stream, true);
+}
+
+speechkv_status speechkv_check_device_error(cudaStream_t stream) {
     DeviceState *s = nullptr;
     speechkv_status st = device_state(&s);
     if (st != SPEECHKV_OK) return st;
-    speechkv::PoolArgs a;
-    a.k_full = k_full;
-    a.v_full = v_full;
-    a.full_off = full_off;
-    a.P = P;
-    a.T = T;
-    a.N = N;
-    a.gate = gate;
-    a.k_cache = k_cache;
-    a.v_cache = v_cache;
-    a.cache_off = cache_off;
-    a.len = len;
-    a.B = B;
-    a.full_rows = full_rows;
-    a.H_kv = H_kv;
-    a.d = d;
-    a.w_eff = layer >= l0 ? w : 1;
-    a.dtype = dtype;
-    a.err = s->err;
-    return speechkv::launch_pool(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
-                                                                       : SPEECHKV_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return SPEECHKV_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpyFromSymbol(&v, speechkv_error_word, sizeof(int)) != cudaSuccess)
+        return SPEECHKV_ERR_CUDA;
+    const int zero = 0;
+    if (v != 0 && cudaMemcpyToSymbol(speechkv_error_word, &zero, sizeof(int)) != cudaSuccess)
+        return SPEECHKV_ERR_CUDA;
+    return static_cast<speechkv_status>(v);
 }
 
 speechkv_status speechkv_pool_hidden(const void *h_full, const int64_t *full_off,
@@ -328,88 +414,6 @@ speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64
                                                                           : SPEECHKV_ERR_CUDA;
 }
 
-speechkv_status speechkv_append(const void *k_new, const void *v_new, void *k_cache,
-                                void *v_cache, const int64_t *cache_off, int32_t *len,
-                                int32_t B, int32_t H_kv, int32_t d, int32_t w, int32_t layer,
-                                int32_t l0, speechkv_dtype dtype, cudaStream_t stream) {
-    if (B < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
-    if (B == 0) return SPEECHKV_OK;
-    if (!k_new || !v_new || !k_cache || !v_cache || !cache_off || !len)
-        return SPEECHKV_ERR_INVALID_ARG;
-    if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_cache, 16) ||
-        !aligned(v_cache, 16) || !aligned(cache_off, 8) || !aligned(len, 4))
-        return SPEECHKV_ERR_INVALID_ARG;
-    DeviceState *s = nullptr;
-    speechkv_status st = device_state(&s);
-    if (st != SPEECHKV_OK) return st;
-    speechkv::AppendArgs a;
-    a.k_new = k_new;
-    a.v_new = v_new;
-    a.k_cache = k_cache;
-    a.v_cache = v_cache;
-    a.cache_off = cache_off;
-    a.len = len;
-    a.B = B;
-    a.H_kv = H_kv;
-    a.d = d;
-    a.dtype = dtype;
-    a.err = s->err;
-    return speechkv::launch_append(a, stream) == cudaSuccess ? SPEECHKV_OK : SPEECHKV_ERR_CUDA;
-}
-
-size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv, int32_t d,
-                                      int32_t grid_ctas) {
-    if (B < 0 || H_kv < 1 || H_q < 1 || H_q % H_kv != 0 || grid_ctas < 0) return 0;
-    if (!speechkv::decode_supported(SPEECHKV_BF16, d, H_q / H_kv)) return 0;
-    int grid = grid_ctas;
-    if (grid == 0) {
-        DeviceState *s = nullptr;
-        if (device_state(&s) != SPEECHKV_OK) return 0;
-        grid = s->num_sms * kAutoCtasPerSmMax;
-    }
-    return workspace_bytes(B, H_q, H_kv, d, grid);
-}
-
-speechkv_status speechkv_decode_attn(const void *q, const void *k_cache, const void *v_cache,
-                                     const int64_t *cache_off, const int32_t *len, void *out,
-                                     float scale, int32_t B, int32_t H_q, int32_t H_kv,
-                                     int32_t d, int32_t w, int32_t layer, int32_t l0,
-                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
-    // the caches and len are only read on this path
-    return decode_common(q, nullptr, nullptr, const_cast<void *>(k_cache),
-                         const_cast<void *>(v_cache), cache_off, const_cast<int32_t *>(len), out,
-                         scale, B, H_q, H_kv, d, w, layer, l0, grid_ctas, workspace,
-                         workspace_bytes_in, dtype, flags, stream, false);
-}
-
-speechkv_status speechkv_decode_step(const void *q, const void *k_new, const void *v_new,
-                                     void *k_cache, void *v_cache, const int64_t *cache_off,
-                                     int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
-                                     int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
-                                     int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                                     speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
-    return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
-                         H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
-                         flags, stream, true);
-}
-
-speechkv_status speechkv_check_device_error(cudaStream_t stream) {
-    DeviceState *s = nullptr;
-    speechkv_status st = device_state(&s);
-    if (st != SPEECHKV_OK) return st;
-    if (cudaStreamSynchronize(stream) != cudaSuccess) return SPEECHKV_ERR_CUDA;
-    int v = 0;
-    if (cudaMemcpyFromSymbol(&v, speechkv_error_word, sizeof(int)) != cudaSuccess)
-        return SPEECHKV_ERR_CUDA;
-    const int zero = 0;
-    if (v != 0 && cudaMemcpyToSymbol(speechkv_error_word, &zero, sizeof(int)) != cudaSuccess)
-        return SPEECHKV_ERR_CUDA;
-    return static_cast<speechkv_status>(v);
-}
-
 }  // extern "C"
 
 // ---------------------------------------------------------------------------
@@ -476,3 +480,105 @@ extern "C" speechkv_status speechkv_decode_step_noalloc(
                          H_kv, d, w, layer, l0, grid, scratch, SPEECHKV_NOALLOC_SCRATCH_BYTES,
                          dtype, flags, stream, true);
 }
+
+extern "C" speechkv_status speechkv_decode_step_paged(
+    const void *q, const void *k_new, const void *v_new, void *k_pages, void *v_pages,
+    const int32_t *block_table, int32_t max_blocks, int32_t block_size, int64_t num_blocks,
+    int32_t *len, void *out, float scale, int32_t B, int32_t H_q, int32_t H_kv, int32_t d,
+    int32_t w, int32_t layer, int32_t l0, int32_t grid_ctas, void *workspace,
+    size_t workspace_bytes_in, speechkv_dtype dtype, uint32_t flags, cudaStream_t stream) {
+    speechkv::CacheMap m;
+    if (B == 0) return SPEECHKV_OK;
+    const speechkv_status st = make_map(block_table, max_blocks, block_size, num_blocks, &m);
+    if (st != SPEECHKV_OK) return st;
+    return decode_common(q, k_new, v_new, k_pages, v_pages, nullptr, len, out, scale, B, H_q,
+                         H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
+                         flags, stream, true, m);
+}
+
+namespace {
+
+speechkv_status pool_impl(const void *k_full, const void *v_full, const int64_t *full_off,
+                              const int32_t *P, const int32_t *T, const int32_t *N,
+                              const float *gate, void *k_cache, void *v_cache,
+                              const int64_t *cache_off, int32_t *len, int32_t B,
+                              int64_t full_rows, int32_t H_kv, int32_t d, int32_t w,
+                              int32_t layer, int32_t l0, speechkv_dtype dtype,
+                              cudaStream_t stream, const speechkv::CacheMap &map) {
+    if (B < 0 || full_rows < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!full_off || !P || !T || !N || !gate || !k_cache || !v_cache ||
+        (!cache_off && !map.table) || !len ||
+        (full_rows > 0 && (!k_full || !v_full)))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(k_full, 16) || !aligned(v_full, 16) || !aligned(k_cache, 16) ||
+        !aligned(v_cache, 16) || !aligned(full_off, 8) || !aligned(cache_off, 8) ||
+        !aligned(P, 4) || !aligned(T, 4) || !aligned(N, 4) || !aligned(len, 4) ||
+        !aligned(gate, 16))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::PoolArgs a;
+    a.k_full = k_full;
+    a.v_full = v_full;
+    a.full_off = full_off;
+    a.P = P;
+    a.T = T;
+    a.N = N;
+    a.gate = gate;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.B = B;
+    a.full_rows = full_rows;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.w_eff = layer >= l0 ? w : 1;
+    a.dtype = dtype;
+    a.err = s->err;
+    a.map = map;
+    return speechkv::launch_pool(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                       : SPEECHKV_ERR_CUDA;
+}
+
+
+
+
+speechkv_status append_impl(const void *k_new, const void *v_new, void *k_cache,
+                                void *v_cache, const int64_t *cache_off, int32_t *len,
+                                int32_t B, int32_t H_kv, int32_t d, int32_t w, int32_t layer,
+                                int32_t l0, speechkv_dtype dtype, cudaStream_t stream,
+                            const speechkv::CacheMap &map) {
+    if (B < 0 || H_kv < 1 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype))
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (d != 64 && d != 128) return SPEECHKV_ERR_UNSUPPORTED;
+    if (B == 0) return SPEECHKV_OK;
+    if (!k_new || !v_new || !k_cache || !v_cache || (!cache_off && !map.table) || !len)
+        return SPEECHKV_ERR_INVALID_ARG;
+    if (!aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_cache, 16) ||
+        !aligned(v_cache, 16) || !aligned(cache_off, 8) || !aligned(len, 4))
+        return SPEECHKV_ERR_INVALID_ARG;
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    speechkv::AppendArgs a;
+    a.k_new = k_new;
+    a.v_new = v_new;
+    a.k_cache = k_cache;
+    a.v_cache = v_cache;
+    a.cache_off = cache_off;
+    a.len = len;
+    a.B = B;
+    a.H_kv = H_kv;
+    a.d = d;
+    a.dtype = dtype;
+    a.err = s->err;
+    a.map = map;
+    return speechkv::launch_append(a, stream) == cudaSuccess ? SPEECHKV_OK : SPEECHKV_ERR_CUDA;
+}
+
+}  // namespace

@@ -25,6 +25,22 @@ __device__ __forceinline__ unsigned long long global_timer_ns() {
 }
 
 // ---------------------------------------------------------------------------
+// cache addressing (contiguous runs or pages; see CacheMap in launch.h)
+// ---------------------------------------------------------------------------
+// Element offset of row t of (request b, KV head h): contiguous runs start
+// at row off_b * H_kv + h * cap_b; pages at ((block * H_kv + h) << bs_log2).
+// -1 when the request's block-table entry for t is not a valid block.
+template <typename Map>
+__device__ __forceinline__ int64_t cache_row(const Map &m, int b, int h, int64_t t, int H_kv,
+                                             int D, int64_t off_b, int64_t cap_b) {
+    if (!m.table) return (off_b * H_kv + (int64_t)h * cap_b + t) * D;
+    const int32_t blk = __ldg(m.table + (int64_t)b * m.max_blocks + (t >> m.bs_log2));
+    if (blk < 0 || blk >= m.num_blocks) return -1;
+    const int64_t in_blk = t & ((1ll << m.bs_log2) - 1);
+    return ((((int64_t)blk * H_kv + h) << m.bs_log2) + in_blk) * D;
+}
+
+// ---------------------------------------------------------------------------
 // element conversions
 // ---------------------------------------------------------------------------
 // bf16 pair packed in a 32-bit word (element 2k in the low half).

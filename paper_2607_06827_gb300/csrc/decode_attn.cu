@@ -133,7 +133,8 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                        const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
                        T *__restrict__ out, float qscale, int B, int H_kv,
                        float *__restrict__ partials, int slot_floats, int *__restrict__ counters,
-                       int *__restrict__ done, int *__restrict__ err, int overlap) {
+                       int *__restrict__ done, int *__restrict__ err, int overlap,
+                       CacheMap map) {
     using C = DecodeCfg<T, D, G>;
     constexpr int W = C::kWarps, S = C::kStages, TR = C::kTileRows, RW = C::kRowsPerWarp;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -166,7 +167,11 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
 
     // ---- 1. per-request lengths (clamped to capacity) and their prefix sums
     for (int b = tid; b < B; b += blockDim.x) {
-        const int64_t o0 = cache_off[b], o1 = cache_off[b + 1];
+        // with pages, every request has the same capacity (max_blocks blocks)
+        // and these offsets only carry it
+        const int64_t capP = (int64_t)map.max_blocks << map.bs_log2;
+        const int64_t o0 = map.table ? (int64_t)b * capP : cache_off[b];
+        const int64_t o1 = map.table ? (int64_t)(b + 1) * capP : cache_off[b + 1];
         const int64_t cap = o1 - o0;
         int64_t L = len[b];
         int32_t nr = -1;
@@ -268,9 +273,12 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                     const int e = (i - tensor * nvec) * kVec;
                     const int hh = e / D, col = e - hh * D;
                     const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
-                    T *dst = (tensor ? vc : kc) + (offs[b] * H_kv + (int64_t)hh * cap + nr) * D +
-                             col;
-                    copy_bytes<16>(dst, src);
+                    const int64_t row = cache_row(map, b, hh, nr, H_kv, D, offs[b], cap);
+                    if (row < 0) {  // invalid page: reported, not written
+                        report_error(err, SPEECHKV_ERR_INVALID_ARG);
+                        continue;
+                    }
+                    copy_bytes<16>((tensor ? vc : kc) + row + col, src);
                 }
             }
         }
@@ -325,6 +333,34 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             const Piece p = piece_at(cum, B, H_kv, u, u1);
             const int64_t cap = offs[p.b + 1] - offs[p.b];
             const int64_t base = offs[p.b] * H_kv + (int64_t)p.h * cap;
+            // Rows [t_from, t_from + nrows) of this (request, head) into the
+            // stage (keys at dst, values kTileBytes further): one bulk copy per
+            // tensor for a contiguous run, one per page segment with a block
+            // table.  An invalid page is reported and read from page 0 instead
+            // (the stage's byte count must still arrive).
+            auto copy_rows = [&](unsigned char *dst, int64_t t_from, int64_t nrows, uint64_t *bar) {
+                if (!map.table) {
+                    const uint32_t bytes = (uint32_t)nrows * C::kRowBytes;
+                    bulk_g2s(dst, kc + (base + t_from) * D, bytes, bar);
+                    bulk_g2s(dst + C::kTileBytes, vc + (base + t_from) * D, bytes, bar);
+                    return;
+                }
+                const int64_t bs = 1ll << map.bs_log2;
+                for (int64_t tt = t_from; tt < t_from + nrows;) {
+                    const int64_t left = t_from + nrows - tt, room = bs - (tt & (bs - 1));
+                    const int64_t seg = left < room ? left : room;
+                    int64_t off = cache_row(map, p.b, p.h, tt, H_kv, D, 0, 0);
+                    if (off < 0) {
+                        report_error(err, SPEECHKV_ERR_INVALID_ARG);
+                        off = 0;
+                    }
+                    const uint32_t at = (uint32_t)(tt - t_from) * C::kRowBytes;
+                    const uint32_t bytes = (uint32_t)seg * C::kRowBytes;
+                    bulk_g2s(dst + at, kc + off, bytes, bar);
+                    bulk_g2s(dst + C::kTileBytes + at, vc + off, bytes, bar);
+                    tt += seg;
+                }
+            };
             // with kAppend, row nr of this (request, head) comes from k_new/v_new
             const int64_t nr = kAppend ? (int64_t)newrow[p.b] : -1;
             for (int64_t t = p.t0; t < p.t1; t += TR) {
@@ -347,17 +383,13 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                     // the tile ends with the new token: cached rows, then one
                     // row from k_new / v_new (always the last row of the run)
                     const uint32_t cached = (uint32_t)(nr - t) * C::kRowBytes;
-                    if (cached) {
-                        bulk_g2s(dst, kc + (base + t) * D, cached, &full_bar[stage]);
-                        bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, cached, &full_bar[stage]);
-                    }
+                    if (cached) copy_rows(dst, t, nr - t, &full_bar[stage]);
                     const int64_t src = ((int64_t)p.b * H_kv + p.h) * D;
                     copy_prior(dst + cached, k_new + src, C::kRowBytes, &full_bar[stage]);
                     copy_prior(dst + C::kTileBytes + cached, v_new + src, C::kRowBytes,
                                &full_bar[stage]);
                 } else {
-                    bulk_g2s(dst, kc + (base + t) * D, bytes, &full_bar[stage]);
-                    bulk_g2s(dst + C::kTileBytes, vc + (base + t) * D, bytes, &full_bar[stage]);
+                    copy_rows(dst, t, rows, &full_bar[stage]);
                 }
                 if (first)
                     copy_prior(dst + 2 * C::kTileBytes, q + ((int64_t)p.b * H_q + p.h * G) * D,
@@ -742,7 +774,7 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
                               static_cast<T *>(a.k_cache), static_cast<T *>(a.v_cache),
                               a.cache_off, a.len, static_cast<T *>(a.out), qscale, a.B, a.H_kv,
                               a.partials, decode_slot_floats(D, G), a.counters, a.done, a.err,
-                              a.overlap ? 1 : 0);
+                              a.overlap ? 1 : 0, a.map);
 }
 
 // Resident CTAs per SM for a batch of B requests (the per-request tables in

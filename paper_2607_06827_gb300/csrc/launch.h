@@ -9,6 +9,18 @@
 
 namespace speechkv {
 
+// Where a layer's cached rows live.  Contiguous (table == nullptr): request
+// b owns rows [cache_off[b], cache_off[b+1]) of every KV head's run, head h
+// of request b starting at row cache_off[b] * H_kv + h * cap_b.  Paged:
+// logical block t >> bs_log2 of request b is physical block
+// table[b * max_blocks + (t >> bs_log2)] of pages [num_blocks][H_kv]
+// [1 << bs_log2][d]; a request's capacity is max_blocks << bs_log2 rows.
+struct CacheMap {
+    const int32_t *table = nullptr;
+    int32_t max_blocks = 0, bs_log2 = 0;
+    int64_t num_blocks = 0;
+};
+
 struct PoolArgs {
     const void *k_full, *v_full;
     const int64_t *full_off;
@@ -22,6 +34,7 @@ struct PoolArgs {
     int32_t H_kv, d, w_eff;
     speechkv_dtype dtype;
     int *err;
+    CacheMap map;  // paged layout when map.table != nullptr (cache_off unused)
 };
 cudaError_t launch_pool(const PoolArgs &a, int num_sms, cudaStream_t stream);
 
@@ -51,6 +64,7 @@ struct AppendArgs {
     int32_t B, H_kv, d;
     speechkv_dtype dtype;
     int *err;
+    CacheMap map;  // paged layout when map.table != nullptr (cache_off unused)
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream);
 
@@ -69,6 +83,7 @@ struct DecodeArgs {
     int *done;         // CTAs past the prologue (fused append only)
     int *err;
     bool overlap;      // SPEECHKV_OVERLAP_PRIOR: start before the previous kernel ends
+    CacheMap map;      // paged layout when map.table != nullptr (cache_off unused)
 };
 
 // Whether (dtype, d, group) has a compiled decode kernel.

@@ -86,14 +86,16 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
                 const int32_t *__restrict__ Ta, const int32_t *__restrict__ Na,
                 const float *__restrict__ gate, T *__restrict__ kc, T *__restrict__ vc,
                 const int64_t *__restrict__ cache_off, int32_t *__restrict__ len,
-                int64_t full_rows, int H_kv, int w, int *__restrict__ err) {
+                int64_t full_rows, int H_kv, int w, CacheMap map, int *__restrict__ err) {
     using C = PoolCfg<T, D>;
     constexpr int EPV = C::kEpv, VH = C::kVecPerHead, HW = C::kHeadsPerWarp, NP = EPV / 2;
     const int b = blockIdx.y;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
     const int64_t row0 = full_off[b], S = full_off[b + 1] - row0;
-    const int64_t base = cache_off[b], cap = cache_off[b + 1] - base;
+    const bool paged = map.table != nullptr;
+    const int64_t base = paged ? 0 : cache_off[b];
+    const int64_t cap = paged ? ((int64_t)map.max_blocks << map.bs_log2) : cache_off[b + 1] - base;
     const int64_t Pb = Pa[b], Tb = Ta[b], Nb = Na[b];
     const int64_t n = (Tb + w - 1) / w;
     const int64_t L = Pb + n + Nb;
@@ -112,9 +114,15 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
     const int64_t VR = (int64_t)H_kv * VH;  // 16-byte vectors per prefill row
     const uint4 *kb = reinterpret_cast<const uint4 *>(kf) + row0 * VR;
     const uint4 *vb = reinterpret_cast<const uint4 *>(vf) + row0 * VR;
-    auto dst_off = [&](int64_t t, int64_t v) {  // element offset of (row t, vector v)
-        const int64_t h = v / VH;
-        return (base * H_kv + h * cap + t) * D + (v - h * VH) * EPV;
+    // element offset of (row t, vector v); -1 when the row's page is invalid
+    auto dst_off = [&](int64_t t, int64_t v) -> int64_t {
+        const int h = (int)(v / VH);
+        const int64_t r = cache_row(map, b, h, t, H_kv, D, base, cap);
+        if (r < 0) {
+            report_error(err, SPEECHKV_ERR_INVALID_ARG);
+            return -1;
+        }
+        return r + (v - (int64_t)h * VH) * EPV;
     };
 
     // ---- copy phase: copy row r is output row r for r < Pc, else the text
@@ -129,10 +137,10 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
         const int64_t dr = Sg / VR, dv = Sg - dr * VR;
         while (r < Ccopy) {
             uint4 kx[kCopyUnroll], vx[kCopyUnroll];
-            int64_t o[kCopyUnroll];  // destination element offset, -1 past the end
+            int64_t o[kCopyUnroll];  // destination element offset, -2 past the end
 #pragma unroll
             for (int k = 0; k < kCopyUnroll; k++) {
-                o[k] = -1;
+                o[k] = -2;
                 if (r < Ccopy) {
                     const bool before = r < Pc;
                     const int64_t src = before ? r : r - Pc + Pb + Tb;  // prefill row
@@ -149,7 +157,8 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
             }
 #pragma unroll
             for (int k = 0; k < kCopyUnroll; k++) {
-                if (o[k] < 0) break;  // the rows of later k are larger
+                if (o[k] == -2) break;  // the rows of later k are larger
+                if (o[k] < 0) continue;  // invalid page (reported)
                 *reinterpret_cast<uint4 *>(kc + o[k]) = kx[k];
                 *reinterpret_cast<uint4 *>(vc + o[k]) = vx[k];
             }
@@ -258,8 +267,10 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
                 ov[2 * k + 1] = av[k].y * inv;
             }
             const int64_t o = dst_off(Pb + i, vi);
-            store_vec<T, EPV>(kc + o, ok);
-            store_vec<T, EPV>(vc + o, ov);
+            if (o >= 0) {
+                store_vec<T, EPV>(kc + o, ok);
+                store_vec<T, EPV>(vc + o, ov);
+            }
         }
     }
 }
@@ -453,7 +464,7 @@ cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t st
     pool_kernel<T, D><<<grid, kPoolThreads, 0, stream>>>(
         static_cast<const T *>(a.k_full), static_cast<const T *>(a.v_full), a.full_off, a.P, a.T,
         a.N, a.gate, static_cast<T *>(a.k_cache), static_cast<T *>(a.v_cache), a.cache_off,
-        a.len, a.full_rows, a.H_kv, a.w_eff, a.err);
+        a.len, a.full_rows, a.H_kv, a.w_eff, a.map, a.err);
     return cudaGetLastError();
 }
 

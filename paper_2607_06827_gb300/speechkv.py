@@ -46,6 +46,15 @@ SIGNATURES = {
                                                     _I32, _I32, _I32, _I32, _I32, _I32,
                                                     _I32, _I32, ctypes.c_int,
                                                     ctypes.c_uint32, _P]),
+    "speechkv_pool_paged": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I32, _I32,
+                                           _I64, _P, _I32, _I64, _I32, _I32, _I32, _I32, _I32,
+                                           ctypes.c_int, _P]),
+    "speechkv_append_paged": (ctypes.c_int, [_P, _P, _P, _P, _P, _I32, _I32, _I64, _P, _I32,
+                                             _I32, _I32, _I32, _I32, _I32, ctypes.c_int, _P]),
+    "speechkv_decode_step_paged": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _I32, _I32, _I64, _P,
+                                                  _P, _F, _I32, _I32, _I32, _I32, _I32, _I32,
+                                                  _I32, _I32, _P, _SZ, ctypes.c_int,
+                                                  ctypes.c_uint32, _P]),
     "speechkv_pool_hidden": (ctypes.c_int, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _I32, _I64,
                                             _I64, _I32, _I32, ctypes.c_int, _P]),
     "speechkv_prefill_attn": (ctypes.c_int, [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _I64, _P, _F,
@@ -197,6 +206,55 @@ def decode_step_noalloc(q, k_new, v_new, k_cache, v_cache, cache_off, length, ou
         _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0, grid_ctas,
         _dtype_code(q), flags, _stream(stream)),
         "speechkv_decode_step_noalloc")
+
+
+def _pages(k_pages, block_table):
+    """(num_blocks, block_size) of pages shaped [num_blocks, H_kv, block_size, d]."""
+    if k_pages.dim() != 4:
+        raise ValueError("pages must be [num_blocks, H_kv, block_size, d]")
+    return k_pages.shape[0], k_pages.shape[2]
+
+
+def pool_paged(k_full, v_full, full_off, P, T, N, gate, k_pages, v_pages, block_table, length,
+               w: int, layer: int, l0: int, stream=None):
+    """speechkv_pool_paged: as pool(), into pages [num_blocks, H_kv,
+    block_size, d] through block_table int32 [B, max_blocks]."""
+    B, max_blocks = block_table.shape
+    full_rows, H_kv, d = k_full.shape
+    nb, bs = _pages(k_pages, block_table)
+    _check(load().speechkv_pool_paged(
+        _ptr(k_full), _ptr(v_full), _ptr(full_off), _ptr(P), _ptr(T), _ptr(N), _ptr(gate),
+        _ptr(k_pages), _ptr(v_pages), _ptr(block_table), max_blocks, bs, nb, _ptr(length), B,
+        full_rows, H_kv, d, w, layer, l0, _dtype_code(k_full), _stream(stream)),
+        "speechkv_pool_paged")
+
+
+def append_paged(k_new, v_new, k_pages, v_pages, block_table, length, w: int, layer: int,
+                 l0: int, stream=None):
+    """speechkv_append_paged: as append(), into pages through block_table."""
+    B, H_kv, d = k_new.shape
+    nb, bs = _pages(k_pages, block_table)
+    _check(load().speechkv_append_paged(
+        _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table),
+        block_table.shape[1], bs, nb, _ptr(length), B, H_kv, d, w, layer, l0,
+        _dtype_code(k_new), _stream(stream)),
+        "speechkv_append_paged")
+
+
+def decode_step_paged(q, k_new, v_new, k_pages, v_pages, block_table, length, out, workspace,
+                      w: int, layer: int, l0: int, scale: float = 0.0, grid_ctas: int = 0,
+                      flags: int = 0, stream=None):
+    """speechkv_decode_step_paged: as decode_step(), over pages through
+    block_table."""
+    B, H_q, d = q.shape
+    H_kv = k_new.shape[1]
+    nb, bs = _pages(k_pages, block_table)
+    _check(load().speechkv_decode_step_paged(
+        _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_pages), _ptr(v_pages), _ptr(block_table),
+        block_table.shape[1], bs, nb, _ptr(length), _ptr(out), float(scale), B, H_q, H_kv, d, w,
+        layer, l0, grid_ctas, _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _dtype_code(q), flags, _stream(stream)),
+        "speechkv_decode_step_paged")
 
 
 def pool_hidden(h_full, full_off, P, T, N, gate, h_out, out_off, length, w: int, stream=None):

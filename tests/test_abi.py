@@ -87,6 +87,16 @@ def test_host_argument_checks_without_gpu():
     assert lib.speechkv_pool_hidden(*ph(0, 2048, 4, sk.BF16)) == sk.OK
     assert lib.speechkv_pool_hidden(*ph(1, 2048, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
     assert lib.speechkv_pool_hidden(*ph(1, 4096, 4, sk.F32)) == sk.ERR_INVALID_ARG   # NULLs
+    # paged caches: block size a power of two, table and page count required
+    pp = lambda B, mb, bs, nb: (*([z] * 9), z, mb, bs, nb, z, B, 10, 8, 128, 4, 0, 0, sk.BF16, z)  # noqa: E731
+    assert lib.speechkv_pool_paged(*pp(0, 4, 64, 8)) == sk.OK
+    assert lib.speechkv_pool_paged(*pp(1, 4, 64, 8)) == sk.ERR_INVALID_ARG        # no table
+    ap = lambda B, bs: (z, z, z, z, z, 4, bs, 8, z, B, 8, 128, 4, 0, 0, sk.BF16, z)  # noqa: E731
+    assert lib.speechkv_append_paged(*ap(0, 64)) == sk.OK
+    assert lib.speechkv_append_paged(*ap(1, 64)) == sk.ERR_INVALID_ARG
+    dp = lambda B: (*([z] * 6), 4, 48, 8, z, z, 0.0, B, 16, 8, 128, 4, 0, 0, 0, z, 0, sk.BF16, 0, z)  # noqa: E731
+    assert lib.speechkv_decode_step_paged(*dp(0)) == sk.OK
+    assert lib.speechkv_decode_step_paged(*dp(1)) == sk.ERR_INVALID_ARG          # no table
     # prefill attention: bf16 and d = 128 only; 32-bit tensor-copy coordinates
     pf = lambda B, q_rows, cache_rows, H_q, H_kv, d, w, dt: (  # noqa: E731
         z, z, q_rows, z, z, z, z, z, z, cache_rows, z, 0.0, B, H_q, H_kv, d, w, 0, 0, dt, z)
