@@ -69,6 +69,8 @@ def parse_args():
     ap.add_argument("--no-unfused", action="store_true",
                     help="skip timing append + decode_attn as two launches")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-paged", action="store_true",
+                    help="skip the paged-cache decode measurement")
     ap.add_argument("--no-prefill", action="store_true",
                     help="skip the prefill-attention measurement")
     ap.add_argument("--prefill-only", action="store_true",
@@ -540,6 +542,100 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
     return res
 
 
+def measure_paged(wl, clocks, block_size: int = 64, steps: int = 64, warmup: int = 4,
+                  chunk: int = 32):
+    """speechkv_decode_step_paged against speechkv_decode_step on the same
+    layer (one pooled, one full-resolution), same inputs: pages of
+    block_size rows in a shuffled block table.  Each path runs `steps` fused
+    steps as CUDA graphs; µs per launch and GB/s of algorithmic bytes."""
+    import numpy as np
+    import torch
+    from paper_2607_06827_gb300 import inputs, speechkv as sk
+    res = {"block_size": block_size, "steps": steps}
+    B, Hq, Hk, d = wl.B, wl.H_q, wl.H_kv, wl.d
+    full_rows = wl.full_rows()
+    full_off = torch.from_numpy(np.concatenate([[0], np.cumsum(full_rows)]).astype(np.int64)).cuda()
+    t32 = lambda x: torch.tensor(x, dtype=torch.int32, device="cuda")  # noqa: E731
+    P, T, N = t32(wl.P), t32(wl.T), t32(wl.N)
+    total = warmup + steps
+    for kind, layer in (("pooled_layer", wl.l0), ("full_layer", 0)):
+        cap = [sk.compressed_len(p, t, n, g, wl.w, layer, wl.l0) + total
+               for p, t, n, g in zip(wl.P, wl.T, wl.N, wl.G)]
+        coff = torch.from_numpy(np.concatenate([[0], np.cumsum(cap)]).astype(np.int64)).cuda()
+        need = [-(-c // block_size) for c in cap]
+        nb, mb = sum(need), max(need)
+        perm = np.random.default_rng(layer).permutation(nb)
+        table = np.full((B, mb), -1, dtype=np.int32)
+        k = 0
+        for b in range(B):
+            table[b, :need[b]] = perm[k:k + need[b]]
+            k += need[b]
+        table = torch.from_numpy(table).cuda()
+        kf = inputs.device_normal((sum(full_rows), Hk, d), torch.bfloat16, "cuda", wl.seed, 50, layer)
+        vf = inputs.device_normal((sum(full_rows), Hk, d), torch.bfloat16, "cuda", wl.seed, 51, layer)
+        gate = inputs.device_normal((Hk, d), torch.float32, "cuda", wl.seed, 52, layer) / math.sqrt(d)
+        kc = torch.empty(sum(cap) * Hk * d, dtype=torch.bfloat16, device="cuda")
+        vc = torch.empty_like(kc)
+        kp = torch.empty((nb, Hk, block_size, d), dtype=torch.bfloat16, device="cuda")
+        vp = torch.empty_like(kp)
+        lc = torch.zeros(B, dtype=torch.int32, device="cuda")
+        lp = torch.zeros(B, dtype=torch.int32, device="cuda")
+        sk.pool(kf, vf, full_off, P, T, N, gate, kc, vc, coff, lc, wl.w, layer, wl.l0)
+        sk.pool_paged(kf, vf, full_off, P, T, N, gate, kp, vp, table, lp, wl.w, layer, wl.l0)
+        del kf, vf
+        for g in range(max(wl.G)):
+            kn = inputs.device_normal((B, Hk, d), torch.bfloat16, "cuda", wl.seed, 53, layer, g)
+            sk.append(kn, kn, kc, vc, coff, lc, wl.w, layer, wl.l0)
+            sk.append_paged(kn, kn, kp, vp, table, lp, wl.w, layer, wl.l0)
+        q = inputs.device_normal((total, B, Hq, d), torch.bfloat16, "cuda", wl.seed, 54, layer)
+        kn = inputs.device_normal((total, B, Hk, d), torch.bfloat16, "cuda", wl.seed, 55, layer)
+        out = torch.empty((B, Hq, d), dtype=torch.bfloat16, device="cuda")
+        ws = sk.new_workspace(B, Hq, Hk, d)
+        rows0 = lc.cpu().tolist()
+
+        def one(paged, s):
+            if paged:
+                sk.decode_step_paged(q[s], kn[s], kn[s], kp, vp, table, lp, out, ws, wl.w,
+                                     layer, wl.l0)
+            else:
+                sk.decode_step(q[s], kn[s], kn[s], kc, vc, coff, lc, out, ws, wl.w, layer, wl.l0)
+        r = {}
+        for paged in (False, True):
+            for s_ in range(warmup):
+                one(paged, s_)
+            torch.cuda.synchronize()
+            graphs = []
+            for c0 in range(warmup, total, chunk):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    for s_ in range(c0, min(total, c0 + chunk)):
+                        one(paged, s_)
+                graphs.append(g)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0 = time.time()
+            e0.record()
+            for g in graphs:
+                g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            clocks and clocks.mark(t0, time.time())
+            r["paged" if paged else "contiguous"] = e0.elapsed_time(e1) * 1e3 / steps
+            del graphs
+        status = sk.check_device_error()
+        assert status == sk.OK, sk.status_string(status)
+        # algorithmic bytes per launch at the middle step (K and V rows read,
+        # q and out, the new row written)
+        rows_mid = sum(rows0) + B * (warmup + steps // 2 + 1)
+        nbytes = rows_mid * Hk * d * 2 * 2 + 2 * B * Hq * d * 2 + B * Hk * d * 2 * 2
+        res[kind] = {"layer": layer, "us_contiguous": round(r["contiguous"], 2),
+                     "us_paged": round(r["paged"], 2),
+                     "gbs_paged": round(nbytes / (r["paged"] * 1e-6) / 1e9, 1),
+                     "paged_over_contiguous": round(r["paged"] / r["contiguous"], 4)}
+        del kc, vc, kp, vp, q, kn, out, ws
+        torch.cuda.empty_cache()
+    return res
+
+
 def measure_hs_pool(wl, clocks, repeats: int = 5, warmup: int = 2, d_model: int = 2048):
     """speechkv_pool_hidden (the HS-compression variant) on the whole prompt
     of the batch: Qwen3-1.7B hidden states (d_model 2048, bf16) pooled with w.
@@ -825,6 +921,9 @@ def main():
                 "speedup_vs_w1_step": (round(w1["step_us"] / r["step_us"], 3) if w1 else None),
             })
 
+    paged = None
+    if not args.no_paged:
+        paged = measure_paged(wl, clocks)
     prefill = None
     if not args.no_prefill:
         prefill = measure_prefill(inputs.qwen_long_audio(args.minutes, args.w), clocks)
@@ -885,6 +984,7 @@ def main():
             } if w1_res else None),
             "by_audio_len": sweep or None,
             "prefill": prefill,
+            "paged": paged,
         }
         print(json.dumps(finite_json(line)), flush=True)
     dist.close()
