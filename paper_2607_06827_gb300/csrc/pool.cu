@@ -278,26 +278,76 @@ __global__ void __launch_bounds__(kPoolThreads, kPoolMinCtas)
 // ---------------------------------------------------------------------------
 // Hidden-state pooling (the HS-compression variant): the same operator on
 // whole hidden vectors, h^_i = sum_j alpha_j h_j with alpha = softmax over the
-// window of gate . h_j.  A CTA of 256 threads handles one output row at a
-// time; each thread owns up to kHsVpt 16-byte vectors of the row, the logits
-// of up to kPoolFrames frames are reduced across the CTA together.
+// window of gate . h_j.
+//
+// One team of kG warps pools one output row at a time, each lane owning up
+// to four 16-byte vectors of the row (a 4 KB bf16 row: four warps), so the
+// logits of a window need one shuffle reduction per frame and a two-value
+// exchange between the team's warps, no CTA-wide barrier.  The input rows
+// stream through shared memory: the team leader copies up to kPoolFrames
+// consecutive rows at a time (a window, a part of a long window, or one kept
+// text row -- always contiguous in the token-major input) with cp.async.bulk
+// into the team's ring of NS stages, completion signalled on an mbarrier per
+// stage.  The team moves a landed stage to registers and the leader refills
+// it at once, before the logits, the window's softmax (running maximum
+// across the parts of a long window, base 2) and the weighted sum in fp32
+// pairs are computed, so the copies in flight cover nearly the whole ring.
+// The CTA holds NT teams; their rings together take most of the SM's shared
+// memory.
 // ---------------------------------------------------------------------------
-constexpr int kHsThreads = 256;
-constexpr int kHsVptMax = 4;  // 16-byte vectors per thread: d_model * sizeof(T) <= 16 KB
+constexpr int kHsMaxWarps = 16;  // 12 for four vectors per lane (registers)
+constexpr int kHsMaxTeams = 8;
+constexpr int kHsMaxStages = 4;
+constexpr int kHsRingBytes = 200 * 1024;  // the teams' rings, one CTA per SM
 
-template <typename T, int kHsVpt>
-__global__ void __launch_bounds__(kHsThreads)
+__device__ __forceinline__ void team_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+// Barrier of a team that also ORs a predicate over its threads.
+__device__ __forceinline__ bool team_any(int id, int nthreads, bool pred) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 q, %1, 0;\n\t"
+        "bar.red.or.pred p, %2, %3, q;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)pred), "r"(id), "r"(nthreads)
+        : "memory");
+    return r != 0;
+}
+
+// Input rows [j, j1) that output row t of a request reads: the window of
+// speech frames for a pooled row, the one kept row otherwise.
+__device__ __forceinline__ bool hs_row_span(int64_t t, int64_t Pb, int64_t Tb, int64_t n, int w,
+                                            int64_t &j, int64_t &j1) {
+    if (t < Pb || t >= Pb + n || w == 1) {
+        j = (t < Pb || w == 1) ? t : t - n + Tb;
+        j1 = j + 1;
+        return true;  // kept as is
+    }
+    j = Pb + (t - Pb) * w;
+    j1 = (j + w < Pb + Tb) ? j + w : Pb + Tb;
+    return false;
+}
+
+template <typename T, int kVpl, int kG>
+__global__ void __launch_bounds__(kVpl >= 4 ? 384 : kHsMaxWarps * 32)
     pool_hidden_kernel(const T *__restrict__ hf, const int64_t *__restrict__ full_off,
                        const int32_t *__restrict__ Pa, const int32_t *__restrict__ Ta,
                        const int32_t *__restrict__ Na, const float *__restrict__ gate,
                        T *__restrict__ ho, const int64_t *__restrict__ out_off,
                        int32_t *__restrict__ len, int64_t full_rows, int64_t out_rows, int VR,
-                       int w, int *__restrict__ err) {
+                       int w, int NT, int NS, int *__restrict__ err) {
     constexpr int EPV = 16 / (int)sizeof(T), NP = EPV / 2;
-    constexpr int kWarps = kHsThreads / 32;
-    __shared__ float red[kPoolFrames][kWarps];
+    constexpr int kTeamThreads = 32 * kG;
+    extern __shared__ __align__(128) unsigned char ring[];
+    __shared__ __align__(8) uint64_t full[kHsMaxTeams * kHsMaxStages];
+    __shared__ float red[kHsMaxTeams][2][kPoolFrames][kG];
     const int b = blockIdx.y;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int team = warp / kG, tw = warp % kG;
 
     const int64_t row0 = full_off[b], S = full_off[b + 1] - row0;
     const int64_t base = out_off[b], cap = out_off[b + 1] - base;
@@ -306,63 +356,130 @@ __global__ void __launch_bounds__(kHsThreads)
     const int64_t L = Pb + n + Nb;
     const bool bad = Pb < 0 || Tb < 0 || Nb < 0 || S != Pb + Tb + Nb || cap < 0 || row0 < 0 ||
                      full_off[b + 1] > full_rows || base < 0 || out_off[b + 1] > out_rows;
-    if (blockIdx.x == 0 && tid == 0) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
         if (bad)
             report_error(err, SPEECHKV_ERR_INVALID_ARG);
         else if (L > cap)
             report_error(err, SPEECHKV_ERR_CAPACITY);
         len[b] = (int32_t)(bad ? 0 : (L < cap ? L : cap));
     }
-    if (bad) return;
+    if (bad) return;  // the whole CTA, before any barrier
     const int64_t rows_out = L < cap ? L : cap;
-    const uint4 *src = reinterpret_cast<const uint4 *>(hf) + row0 * VR;
-    uint4 *dst = reinterpret_cast<uint4 *>(ho) + base * VR;
+    const uint32_t row_bytes = (uint32_t)VR * 16u;
+    const uint32_t stage_bytes = kPoolFrames * row_bytes;
 
-    // the thread's slice of the gate, scaled by log2(e) (softmax in base 2)
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < NT * NS; s++) mbar_init(&full[s], 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (team >= NT) return;
+
+    unsigned char *tring = ring + (size_t)team * NS * stage_bytes;
+    uint64_t *tfull = full + team * NS;
+    const int bar_id = 1 + team;  // named barrier of the team (kG > 1)
+    const bool leader = tw == 0 && lane == 0;
+    const int64_t R = (int64_t)gridDim.x * NT;  // teams working on this request
+    const int64_t first = (int64_t)blockIdx.x * NT + team;
+    const unsigned char *src = reinterpret_cast<const unsigned char *>(hf) + row0 * (int64_t)row_bytes;
+
+    // The leader's copy pointer runs NS chunks ahead of the team.
+    int64_t pt = first, pj = 0, pj1 = 0;
+    if (pt < rows_out) hs_row_span(pt, Pb, Tb, n, w, pj, pj1);
+    int ps = 0;
+    auto issue = [&]() {
+        if (pt >= rows_out) return;
+        const int nf = pj1 - pj < kPoolFrames ? (int)(pj1 - pj) : kPoolFrames;
+        mbar_arrive_expect_tx(&tfull[ps], (uint32_t)nf * row_bytes);
+        bulk_g2s(tring + (size_t)ps * stage_bytes, src + pj * (int64_t)row_bytes,
+                 (uint32_t)nf * row_bytes, &tfull[ps]);
+        if (++ps == NS) ps = 0;
+        pj += kPoolFrames;
+        if (pj >= pj1) {
+            pt += R;
+            if (pt < rows_out) hs_row_span(pt, Pb, Tb, n, w, pj, pj1);
+        }
+    };
+    int64_t n_issued = 0, n_done = 0;
+    if (leader)
+        for (int s = 0; s < NS && pt < rows_out; s++) {
+            issue();
+            n_issued++;
+        }
+
+    // the lane's vectors of the row: vec(x) = tw * 32 * kVpl + x * 32 + lane
+    const int vbase = tw * 32 * kVpl + lane;
     constexpr float kLog2e = 1.4426950408889634f;
-    float2 u[kHsVpt][NP];
+    float2 u[kVpl][NP];
 #pragma unroll
-    for (int x = 0; x < kHsVpt; x++) {
-        const int v = tid + x * kHsThreads;
+    for (int x = 0; x < kVpl; x++) {
+        const int v = vbase + x * 32;
 #pragma unroll
-        for (int k = 0; k < NP; k++) {
+        for (int k = 0; k < NP; k++)
             u[x][k] = v < VR ? make_float2(gate[v * EPV + 2 * k] * kLog2e,
                                            gate[v * EPV + 2 * k + 1] * kLog2e)
                              : make_float2(0.f, 0.f);
-        }
     }
+    uint4 *dst = reinterpret_cast<uint4 *>(ho) + base * (int64_t)VR;
 
-    for (int64_t t = blockIdx.x; t < rows_out; t += gridDim.x) {
-        if (t < Pb || t >= Pb + n || w == 1) {
-            // text row (or no pooling): bit-exact copy
-            const int64_t s = (t < Pb || w == 1) ? t : t - n + Tb;
-#pragma unroll
-            for (int x = 0; x < kHsVpt; x++) {
-                const int v = tid + x * kHsThreads;
-                if (v < VR) dst[t * VR + v] = __ldcs(src + s * VR + v);
-            }
-            continue;
-        }
-        const int64_t j0 = Pb + (t - Pb) * w;
-        const int64_t j1 = (j0 + w < Pb + Tb) ? j0 + w : Pb + Tb;
+    int sc = 0;        // stage of the next chunk
+    uint32_t ph = 0;   // its phase parity
+    int rb = 0;        // red[] buffer of the next exchange (kG > 1)
+    bool stop = false;
+    for (int64_t t = first; t < rows_out && !stop; t += R) {
+        int64_t j, j1;
+        const bool kept = hs_row_span(t, Pb, Tb, n, w, j, j1);
         float m = -INFINITY, l = 0.f;
-        float2 acc[kHsVpt][NP];
+        float2 acc[kVpl][NP];
 #pragma unroll
-        for (int x = 0; x < kHsVpt; x++)
+        for (int x = 0; x < kVpl; x++)
 #pragma unroll
             for (int k = 0; k < NP; k++) acc[x][k] = make_float2(0.f, 0.f);
-        for (int64_t j = j0; j < j1; j += kPoolFrames) {
+        for (; j < j1; j += kPoolFrames) {
             const int nf = j1 - j < kPoolFrames ? (int)(j1 - j) : kPoolFrames;
-            uint4 raw[kPoolFrames][kHsVpt];
+            const bool landed = mbar_wait_bounded(&tfull[sc], ph, err);
+            const uint4 *st = reinterpret_cast<const uint4 *>(tring + (size_t)sc * stage_bytes);
+            uint4 raw[kPoolFrames][kVpl];
+#pragma unroll
+            for (int f = 0; f < kPoolFrames; f++)
+#pragma unroll
+                for (int x = 0; x < kVpl; x++) {
+                    const int v = vbase + x * 32;
+                    raw[f][x] = (landed && f < nf && v < VR) ? st[f * VR + v]
+                                                             : make_uint4(0u, 0u, 0u, 0u);
+                }
+            // one barrier: every thread of the team has its words (the stage
+            // may be refilled) and every thread's wait succeeded
+            const bool failed = kG > 1 ? team_any(bar_id, kTeamThreads, !landed)
+                                       : !__all_sync(0xffffffffu, landed);
+            if (failed) {
+                stop = true;
+                break;
+            }
+            n_done++;
+            if (leader && pt < rows_out) {
+                issue();
+                n_issued++;
+            }
+            if (++sc == NS) {
+                sc = 0;
+                ph ^= 1;
+            }
+            if (kept) {
+                // text row (or no pooling): bit-exact copy
+#pragma unroll
+                for (int x = 0; x < kVpl; x++) {
+                    const int v = vbase + x * 32;
+                    if (v < VR) __stcs(dst + t * VR + v, raw[0][x]);
+                }
+                continue;
+            }
             float z[kPoolFrames];
 #pragma unroll
             for (int f = 0; f < kPoolFrames; f++) {
                 float2 a2 = make_float2(0.f, 0.f);
 #pragma unroll
-                for (int x = 0; x < kHsVpt; x++) {
-                    const int v = tid + x * kHsThreads;
-                    raw[f][x] = (f < nf && v < VR) ? __ldcs(src + (j + f) * VR + v)
-                                                   : make_uint4(0u, 0u, 0u, 0u);
+                for (int x = 0; x < kVpl; x++) {
                     float2 e[NP];
                     widen2<T>(raw[f][x], e);
 #pragma unroll
@@ -370,46 +487,56 @@ __global__ void __launch_bounds__(kHsThreads)
                 }
                 z[f] = warp_sum(a2.x + a2.y);
             }
-            // CTA-wide sums of the frames' logits (fixed order: deterministic)
-            if (lane == 0)
+            if (kG > 1) {
+                // the team's warps exchange their partial logits (fixed
+                // order); red[] alternates between two buffers, so the
+                // barriers of the next chunk separate these reads from the
+                // next writes of the buffer
+                if (lane == 0)
 #pragma unroll
-                for (int f = 0; f < kPoolFrames; f++) red[f][warp] = z[f];
-            __syncthreads();
+                    for (int f = 0; f < kPoolFrames; f++) red[team][rb][f][tw] = z[f];
+                team_sync(bar_id, kTeamThreads);
+#pragma unroll
+                for (int f = 0; f < kPoolFrames; f++) {
+                    float zz = 0.f;
+#pragma unroll
+                    for (int g = 0; g < kG; g++) zz += red[team][rb][f][g];
+                    z[f] = zz;
+                }
+                rb ^= 1;
+            }
             float mb = m;
 #pragma unroll
-            for (int f = 0; f < kPoolFrames; f++) {
-                float zz = 0.f;
-#pragma unroll
-                for (int x = 0; x < kWarps; x++) zz += red[f][x];
-                z[f] = zz;
-                if (f < nf) mb = fmaxf(mb, zz);
-            }
-            __syncthreads();  // red[] is rewritten by the next frames
+            for (int f = 0; f < kPoolFrames; f++)
+                if (f < nf) mb = fmaxf(mb, z[f]);
             const float corr = fast_exp2(m - mb);  // 0 on the first frames
             l *= corr;
 #pragma unroll
-            for (int x = 0; x < kHsVpt; x++)
+            for (int x = 0; x < kVpl; x++)
 #pragma unroll
                 for (int k = 0; k < NP; k++) acc[x][k] = fmul2(acc[x][k], make_float2(corr, corr));
 #pragma unroll
             for (int f = 0; f < kPoolFrames; f++) {
-                if (f >= nf) break;
-                const float p = fast_exp2(z[f] - mb);
-                l += p;
+                if (f < nf) {
+                    const float p = fast_exp2(z[f] - mb);
+                    l += p;
 #pragma unroll
-                for (int x = 0; x < kHsVpt; x++) {
-                    float2 e[NP];
-                    widen2_prmt<T>(raw[f][x], e);
+                    for (int x = 0; x < kVpl; x++) {
+                        float2 e[NP];
+                        widen2_prmt<T>(raw[f][x], e);
 #pragma unroll
-                    for (int k = 0; k < NP; k++) acc[x][k] = ffma2(make_float2(p, p), e[k], acc[x][k]);
+                        for (int k = 0; k < NP; k++)
+                            acc[x][k] = ffma2(make_float2(p, p), e[k], acc[x][k]);
+                    }
                 }
             }
             m = mb;
         }
+        if (stop || kept) continue;
         const float inv = 1.f / l;
 #pragma unroll
-        for (int x = 0; x < kHsVpt; x++) {
-            const int v = tid + x * kHsThreads;
+        for (int x = 0; x < kVpl; x++) {
+            const int v = vbase + x * 32;
             if (v >= VR) continue;
             float o[EPV];
 #pragma unroll
@@ -420,29 +547,83 @@ __global__ void __launch_bounds__(kHsThreads)
             store_vec<T, EPV>(reinterpret_cast<T *>(dst + t * VR + v), o);
         }
     }
+    if (stop && leader) {
+        // the copies still in flight land before the CTA's shared memory
+        // goes away
+        for (int64_t k = n_done; k < n_issued; k++) {
+            mbar_wait_bounded(&tfull[sc], ph, err);
+            if (++sc == NS) {
+                sc = 0;
+                ph ^= 1;
+            }
+        }
+    }
 }
 
-template <typename T, int VPT>
-cudaError_t launch_pool_hidden_vpt(const PoolHiddenArgs &a, const dim3 &grid, int VR,
+// Vectors per lane and warps per team for rows of VR 16-byte vectors; the
+// teams per CTA and stages per team that fit the ring budget.
+struct HsPlan {
+    int vpl, g, nt, ns;
+};
+inline HsPlan hs_plan(int VR) {
+    HsPlan p;
+    // two vectors per lane up to 4 KB rows (teams of up to four warps, up
+    // to 16 warps per CTA), four for wider rows (registers: 12 warps)
+    p.vpl = VR <= 32 ? 1 : VR <= 256 ? 2 : 4;
+    p.g = (VR + 32 * p.vpl - 1) / (32 * p.vpl);
+    const int max_warps = p.vpl >= 4 ? 12 : kHsMaxWarps;
+    const int64_t stage = (int64_t)kPoolFrames * VR * 16;
+    const int slots = (int)(kHsRingBytes / stage);  // >= 3 for rows of up to 16 KB
+    // as many teams as the warp budget allows with two stages each, then
+    // the stages that the ring budget leaves for each team
+    p.nt = slots / 2;
+    if (p.nt > kHsMaxTeams) p.nt = kHsMaxTeams;
+    if (p.nt > max_warps / p.g) p.nt = max_warps / p.g;
+    if (p.nt < 1) p.nt = 1;
+    p.ns = slots / p.nt;
+    if (p.ns > kHsMaxStages) p.ns = kHsMaxStages;
+    return p;
+}
+
+template <typename T, int kVpl, int kG>
+cudaError_t launch_pool_hidden_cfg(const PoolHiddenArgs &a, const HsPlan &p, int num_sms, int VR,
                                    cudaStream_t stream) {
-    pool_hidden_kernel<T, VPT><<<grid, kHsThreads, 0, stream>>>(
+    auto kern = pool_hidden_kernel<T, kVpl, kG>;
+    static int configured_device_mask = 0;  // devices with the smem attribute set
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (!(dev < 31 && (__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev)))) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kHsRingBytes);
+        if (e != cudaSuccess) return e;
+        if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
+    }
+    int64_t x = ((int64_t)num_sms + a.B - 1) / a.B;  // one CTA per SM over the batch
+    if (x < 1) x = 1;
+    if (x > 65535) x = 65535;
+    const dim3 grid((unsigned)x, (unsigned)a.B);
+    const size_t smem = (size_t)p.nt * p.ns * kPoolFrames * VR * 16;
+    kern<<<grid, p.nt * kG * 32, smem, stream>>>(
         static_cast<const T *>(a.h_full), a.full_off, a.P, a.T, a.N, a.gate,
-        static_cast<T *>(a.h_out), a.out_off, a.len, a.full_rows, a.out_rows, VR, a.w, a.err);
+        static_cast<T *>(a.h_out), a.out_off, a.len, a.full_rows, a.out_rows, VR, a.w, p.nt, p.ns,
+        a.err);
     return cudaGetLastError();
 }
 
 template <typename T>
 cudaError_t launch_pool_hidden_instance(const PoolHiddenArgs &a, int num_sms,
                                         cudaStream_t stream) {
-    int64_t x = ((int64_t)4 * num_sms + a.B - 1) / a.B;
-    if (x < 1) x = 1;
-    if (x > 65535) x = 65535;
-    const dim3 grid((unsigned)x, (unsigned)a.B);
     const int VR = (int)((int64_t)a.d_model * (int64_t)sizeof(T) / 16);
-    const int vpt = (VR + kHsThreads - 1) / kHsThreads;
-    if (vpt <= 1) return launch_pool_hidden_vpt<T, 1>(a, grid, VR, stream);
-    if (vpt <= 2) return launch_pool_hidden_vpt<T, 2>(a, grid, VR, stream);
-    return launch_pool_hidden_vpt<T, kHsVptMax>(a, grid, VR, stream);
+    const HsPlan p = hs_plan(VR);
+    if (p.vpl == 4)
+        return p.g == 8 ? launch_pool_hidden_cfg<T, 4, 8>(a, p, num_sms, VR, stream)
+                        : launch_pool_hidden_cfg<T, 4, 4>(a, p, num_sms, VR, stream);
+    if (p.vpl == 2) {
+        if (p.g == 4) return launch_pool_hidden_cfg<T, 2, 4>(a, p, num_sms, VR, stream);
+        if (p.g == 2) return launch_pool_hidden_cfg<T, 2, 2>(a, p, num_sms, VR, stream);
+        return launch_pool_hidden_cfg<T, 2, 1>(a, p, num_sms, VR, stream);
+    }
+    return launch_pool_hidden_cfg<T, 1, 1>(a, p, num_sms, VR, stream);
 }
 
 template <typename T, int D>
@@ -472,7 +653,7 @@ cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t st
 
 bool pool_hidden_supported(speechkv_dtype dtype, int d_model) {
     const int es = dtype == SPEECHKV_F32 ? 4 : 2;
-    return d_model > 0 && (d_model * es) % 16 == 0 && d_model * es <= kHsVptMax * kHsThreads * 16;
+    return d_model > 0 && (d_model * es) % 16 == 0 && d_model * es <= 16 * 1024;  // rows of up to 16 KB
 }
 
 cudaError_t launch_pool_hidden(const PoolHiddenArgs &a, int num_sms, cudaStream_t stream) {

@@ -79,6 +79,26 @@ def test_hs_pool_fp32(oracle, d_model):
     _check(oracle, wl, d_model, hs, gate, out, out_off, ln)
 
 
+@pytest.mark.parametrize("d_model,w", [(256, 4), (512, 3), (1024, 4), (4096, 4), (8192, 5)])
+def test_hs_pool_bf16_row_widths(oracle, d_model, w):
+    """Rows of 0.5 to 16 KB (one to four vectors per lane, teams of one to
+    eight warps); w = 5 splits every window into a full group of frames and
+    a ragged one."""
+    wl = _wl(P=(2, 0), T=(151, 64), N=(3, 9), w=w, seed=3005)
+    sk, hs, gate, out, out_off, ln = _run(wl, d_model)
+    assert sk.check_device_error() == sk.OK
+    _check(oracle, wl, d_model, hs, gate, out, out_off, ln)
+
+
+def test_hs_pool_long_requests(oracle):
+    """Requests long enough that every CTA pools many rows (the staging
+    ring of each CTA is reused many times over)."""
+    wl = _wl(P=(0, 9), T=(30000, 7001), N=(64, 3), w=4, seed=3006)
+    sk, hs, gate, out, out_off, ln = _run(wl, 2048)
+    assert sk.check_device_error() == sk.OK
+    _check(oracle, wl, 2048, hs, gate, out, out_off, ln)
+
+
 def test_hs_pool_peaked_gate(oracle):
     """A gate sixteen times larger: near-one-hot weights in every window."""
     wl = _wl(w=4, seed=3003)
