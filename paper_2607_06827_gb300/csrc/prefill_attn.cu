@@ -7,20 +7,27 @@
 // and sees rows 0 .. pi(t) (causality over the compressed sequence).
 //
 // Blackwell tensor-core flash attention, bf16 in, fp32 accumulate, d = 128:
-//   * persistent: one CTA per SM walks work items (request, query head,
-//     128-row query tile) ordered by (request, KV head), so that the CTAs
-//     running together read the same keys and values (from L2);
-//   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the query tile
-//     and of 128-row key and value tiles (two stages) from the cache;
-//   * warp 1 lane 0: tcgen05.mma issue -- S = Q K^T into a 128-column TMEM
-//     buffer, O += P V into another, with P read from TMEM (two 64-column
-//     buffers) and V as the MN-major shared-memory operand;
-//   * warps 2-5: softmax, one query row per thread (= TMEM lane): the S row
-//     read from TMEM in one load (S is then free for the next Q K^T), row
-//     maximum, base-2 exponentials with log2(e)/sqrt(d) folded in, P stored
-//     as bf16 pairs into its TMEM buffer, O rescaled in TMEM only when a
-//     row's maximum rose by more than 2^8 (lazy rescaling), and the epilogue
-//     O / l to global memory.
+//   * persistent: one CTA per SM walks work items (request, KV head, 128-row
+//     query tile, pair of query heads of that KV head) ordered by (request,
+//     KV head), so that the CTAs running together read the same keys and
+//     values (from L2); the two query tiles of an item ("slots") share every
+//     key and value tile, which halves the L2 -> SM traffic per FLOP (at one
+//     query tile per CTA the loads, not the tensor cores, set the pace);
+//   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the two query
+//     tiles and of 128-row key tiles (three stages) and value tiles (two
+//     stages), keys one tile ahead of values;
+//   * warp 1 lane 0: tcgen05.mma issue -- per key tile and slot x,
+//     O_x += P_x V then S_x = Q_x K^T of the next key tile, into 128-column
+//     TMEM buffers (S_0, S_1, O_0, O_1: all 512 columns); P_x is stored over
+//     the first half of S_x and read as the A operand from TMEM, so a slot's
+//     next Q K^T waits for its P V while the other slot's products keep the
+//     tensor pipe busy;
+//   * warps 2-5 (slot 0) and 6-9 (slot 1): softmax, one query row per thread
+//     (= TMEM lane): the S row read from TMEM in one load, masked keys set to
+//     -inf once per masked tile, row maximum, base-2 exponentials with
+//     log2(e)/sqrt(d) folded in, P stored as bf16 pairs, O rescaled in TMEM
+//     only when a row's maximum rose by more than 2^8 (lazy rescaling), and
+//     the epilogue O / l to global memory.
 // Cache rows past a request's compressed length are zeroed in the value
 // stage (their contents are unspecified and the MMA would multiply them by
 // zero weights: 0 x NaN is NaN).  Every wait is bounded; on a timeout the CTA
@@ -39,34 +46,68 @@ namespace {
 constexpr int kBM = 128;  // query rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per tile
 constexpr int kD = 128;   // head dimension
-constexpr int kThreads = 192;
+constexpr int kSlots = 2;    // query tiles per CTA (two query heads of one KV head)
+constexpr int kThreads = 64 + kSlots * 128;  // TMA warp, MMA warp, a softmax warpgroup per slot
 constexpr int kTileBytes = kBM * kD * 2;  // one bf16 tile of 128 rows x 128
 constexpr int kHalf = kTileBytes / 2;     // its 64-column block (128-byte rows)
-constexpr int kStages = 2;                // key/value ring
-constexpr uint32_t kTmemCols = 512;       // S: 0..127, O: 128..255, P: 256..319 and 320..383
+constexpr int kKStages = 3;               // key ring
+constexpr int kVStages = 2;               // value ring
+constexpr uint32_t kTmemCols = 512;       // S_x: 128 x, O_x: 256 + 128 x; P_x over S_x's first 64
 
 // shared memory (offsets from a 1024-byte aligned base)
 constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kTileBytes;
-constexpr int kOffV = kOffK + kStages * kTileBytes;
-constexpr int kOffBar = kOffV + kStages * kTileBytes;
-enum Bar { kQFull, kQEmpty, kKFull, kVFull = kKFull + kStages, kKEmpty = kVFull + kStages,
-           kVEmpty = kKEmpty + kStages, kSFull = kVEmpty + kStages, kSFree,
-           kPFull,                // [2]: P of tile g is in TMEM buffer g & 1
-           kPFree = kPFull + 2,   // [2]: the P V that read buffer g & 1 is done
-           kDrain = kPFree + 2, kNumBars };
+constexpr int kOffK = kOffQ + kSlots * kTileBytes;
+constexpr int kOffV = kOffK + kKStages * kTileBytes;
+constexpr int kOffBar = kOffV + kVStages * kTileBytes;
+enum Bar { kQFull, kQEmpty = kQFull + kSlots, kKFull = kQEmpty + kSlots,
+           kKEmpty = kKFull + kKStages, kVFull = kKEmpty + kKStages,
+           kVEmpty = kVFull + kVStages,
+           kSFull = kVEmpty + kVStages,  // [slot]: S_x = Q_x K^T is in TMEM
+           kPFull = kSFull + kSlots,     // [slot]: P_x is in TMEM (the slot's 128 threads)
+           kODone = kPFull + kSlots,     // [slot]: O_x += P_x V is done
+           kDrain = kODone + kSlots, kNumBars };
 constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem address, abort flag, largest tile count
-constexpr int kOffTab = kOffMisc + 16;
 
-struct Req {         // per-request table in shared memory
+struct Req {         // one request's geometry, from the argument arrays
     int64_t q0;      // first query row
     int64_t kv0;     // cache_off[b]
     int64_t cap;     // capacity (rows)
     int32_t P, T, N, n, S, tiles;
 };
-static_assert(sizeof(Req) == 48, "table entry");
 
-size_t smem_bytes(int B) { return (size_t)kOffTab + (size_t)B * sizeof(Req) + 1024; }
+constexpr size_t kSmemBytes = (size_t)kOffMisc + 16 + 1024;  // + alignment of the base
+static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
+
+// Request b's table entry, read from the argument arrays (cached in L1);
+// tiles = 0 marks a request that is skipped.  *bad: 1 inconsistent, 2 the
+// compressed rows exceed the capacity.
+struct ReqSrc {
+    const int64_t *q_off, *cache_off;
+    const int32_t *P, *T, *N;
+    int64_t q_rows, cache_rows;
+    int w;
+    __device__ __forceinline__ Req operator()(int b, int *bad = nullptr) const {
+        Req q;
+        q.q0 = q_off[b];
+        const int64_t q1 = q_off[b + 1];
+        q.kv0 = cache_off[b];
+        const int64_t kv1 = cache_off[b + 1];
+        q.cap = kv1 - q.kv0;
+        q.P = P[b];
+        q.T = T[b];
+        q.N = N[b];
+        q.n = q.T >= 0 ? (int32_t)(((int64_t)q.T + w - 1) / w) : 0;
+        const int64_t S = (int64_t)q.P + q.T + q.N;
+        const int64_t c = (int64_t)q.P + q.n + q.N;
+        q.S = (int32_t)S;
+        const bool ok = q.P >= 0 && q.T >= 0 && q.N >= 0 && q.q0 >= 0 && q1 - q.q0 == S &&
+                        q1 <= q_rows && q.kv0 >= 0 && kv1 <= cache_rows && S < (1ll << 31);
+        const int why = !ok ? 1 : (c > q.cap ? 2 : 0);
+        if (bad) *bad = why;
+        q.tiles = why == 0 ? (int32_t)((S + kBM - 1) / kBM) : 0;
+        return q;
+    }
+};
 
 __device__ __forceinline__ int64_t pi_of(const Req &q, int64_t t, int w) {
     if (t < q.P) return t;
@@ -176,25 +217,42 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t parity, volatil
     }
 }
 
+// Non-blocking check that the phase with the given parity has completed.
+__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Work item k of the CTA-independent order: (request, KV head) outermost,
-// then query tiles from the last down, then the query heads of the KV head's
-// group.  CTAs working at the same time share one (request, KV head)'s keys
-// and values, which stay in L2 while they are read again and again.
+// then query tiles from the last down, then groups of up to kSlots query
+// heads of the KV head's group (they share every key and value tile).  CTAs
+// working at the same time share one (request, KV head)'s keys and values.
 struct Item {
-    int b, hq, i;
+    int b, hq0, n, i;  // request, first query head, heads (slots used), query tile
     bool valid;
 };
-__device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int B, int H_q, int H_kv,
-                                        const Req *tab) {
+__device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int H_q, int H_kv,
+                                        const ReqSrc &tab, Req &q) {
     Item it;
     const int G = H_q / H_kv;
-    const int64_t per = (int64_t)tiles_max * G;  // items of one (request, KV head)
+    const int ng = (G + kSlots - 1) / kSlots;    // head groups of a KV head
+    const int64_t per = (int64_t)tiles_max * ng;  // items of one (request, KV head)
     const int bh = (int)(k / per);
     const int rem = (int)(k - (int64_t)bh * per);
     it.b = bh / H_kv;
-    it.hq = (bh - it.b * H_kv) * G + rem % G;
-    it.i = tiles_max - 1 - rem / G;
-    it.valid = it.i < tab[it.b].tiles;
+    const int grp = rem % ng;
+    it.hq0 = (bh - it.b * H_kv) * G + grp * kSlots;
+    it.n = min(kSlots, G - grp * kSlots);
+    it.i = tiles_max - 1 - rem / ng;
+    q = tab(it.b);
+    it.valid = it.i < q.tiles;
     return it;
 }
 
@@ -214,25 +272,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
     volatile int *abort = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
     int *tiles_max_s = reinterpret_cast<int *>(sm + kOffMisc + 8);
-    Req *tab = reinterpret_cast<Req *>(sm + kOffTab);
+    const ReqSrc tab{q_off, cache_off, Pa, Ta, Na, q_rows, cache_rows, w};
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = H_q / H_kv;
 
-    // ---- prologue: barriers, TMEM, per-request table
+    // ---- prologue: barriers, TMEM, largest tile count
     if (tid == 0) {
-        mbar_init(&bar[kQFull], 1);
-        mbar_init(&bar[kQEmpty], 1);
-        for (int s = 0; s < kStages; s++) {
-            mbar_init(&bar[kKFull + s], 1);
-            mbar_init(&bar[kVFull + s], 1);
-            mbar_init(&bar[kKEmpty + s], 1);
-            mbar_init(&bar[kVEmpty + s], 1);
-        }
-        mbar_init(&bar[kSFull], 1);
-        mbar_init(&bar[kSFree], kBM);
-        for (int x = 0; x < 2; x++) {
+        for (int x = 0; x < kSlots; x++) {
+            mbar_init(&bar[kQFull + x], 1);
+            mbar_init(&bar[kQEmpty + x], 1);
+            mbar_init(&bar[kSFull + x], 1);
             mbar_init(&bar[kPFull + x], kBM);
-            mbar_init(&bar[kPFree + x], 1);
+            mbar_init(&bar[kODone + x], 1);
+        }
+        for (int s = 0; s < kKStages; s++) {
+            mbar_init(&bar[kKFull + s], 1);
+            mbar_init(&bar[kKEmpty + s], 1);
+        }
+        for (int s = 0; s < kVStages; s++) {
+            mbar_init(&bar[kVFull + s], 1);
+            mbar_init(&bar[kVEmpty + s], 1);
         }
         mbar_init(&bar[kDrain], 1);
         fence_mbar_init();
@@ -246,35 +305,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    for (int b = tid; b < B; b += kThreads) {
-        Req q;
-        q.q0 = q_off[b];
-        const int64_t q1 = q_off[b + 1];
-        q.kv0 = cache_off[b];
-        const int64_t kv1 = cache_off[b + 1];
-        q.cap = kv1 - q.kv0;
-        q.P = Pa[b];
-        q.T = Ta[b];
-        q.N = Na[b];
-        q.n = q.T >= 0 ? (int32_t)(((int64_t)q.T + w - 1) / w) : 0;
-        const int64_t S = (int64_t)q.P + q.T + q.N;
-        const int64_t c = (int64_t)q.P + q.n + q.N;
-        q.S = (int32_t)S;
-        bool ok = q.P >= 0 && q.T >= 0 && q.N >= 0 && q.q0 >= 0 && q1 - q.q0 == S &&
-                  q1 <= q_rows && q.kv0 >= 0 && kv1 <= cache_rows && S < (1ll << 31);
-        if (!ok) {
-            if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
-        } else if (c > q.cap) {
-            if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_CAPACITY);
-            ok = false;
-        }
-        q.tiles = ok ? (int32_t)((S + kBM - 1) / kBM) : 0;
-        tab[b] = q;
-    }
-    __syncthreads();
     if (warp == 0) {
+        // largest tile count over the batch; CTA 0 reports the skipped requests
         int mx = 0;
-        for (int b = lane; b < B; b += 32) mx = max(mx, tab[b].tiles);
+        for (int b = lane; b < B; b += 32) {
+            int bad = 0;
+            mx = max(mx, tab(b, &bad).tiles);
+            if (bad && blockIdx.x == 0)
+                report_error(err, bad == 1 ? SPEECHKV_ERR_INVALID_ARG : SPEECHKV_ERR_CAPACITY);
+        }
         for (int o = 16; o > 0; o >>= 1) mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
         if (lane == 0) *tiles_max_s = mx;
     }
@@ -283,128 +322,178 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
     const int tiles_max = *tiles_max_s;
-    const int64_t total = (int64_t)tiles_max * B * H_q;
-
+    const int ng = (G + kSlots - 1) / kSlots;
+    const int64_t total = (int64_t)tiles_max * B * H_kv * ng;
     unsigned char *sQ = sm + kOffQ, *sK = sm + kOffK, *sV = sm + kOffV;
 
     if (warp == 0) {
         // ===================== TMA producer =====================
+        // One stream of copies over the CTA's items: the query tiles of an
+        // item (one buffer per slot), then its key and value tiles with the
+        // keys one tile ahead of the values (a value tile waits for an older
+        // P V than the key tile issued before it).
         if (lane == 0) {
-            int64_t it = 0, g = 0;
-            bool k_only = false;
-            for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
-                const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
+            int64_t uq[kSlots] = {}, gk = 0, gv = 0;  // query (per slot), key, value tiles issued
+            int pend_y = -1;                          // cache row of the value tile still to issue
+            bool stop = false;
+            auto issue_v = [&](int y) -> bool {
+                const int s = (int)(gv % kVStages);
+                const int64_t u = gv / kVStages;
+                if (gv >= kVStages && !wait_bar(&bar[kVEmpty + s], (uint32_t)((u - 1) & 1), abort, err))
+                    return false;
+                mbar_arrive_expect_tx(&bar[kVFull + s], kTileBytes);
+                tma_2d(sV + s * kTileBytes, &tm_v, 0, y, &bar[kVFull + s]);
+                tma_2d(sV + s * kTileBytes + kHalf, &tm_v, 64, y, &bar[kVFull + s]);
+                ++gv;
+                return true;
+            };
+            for (int64_t k = blockIdx.x; k < total && !stop && !*abort; k += gridDim.x) {
+                Req q;
+                const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
                 if (!item.valid) continue;
-                const Req &q = tab[item.b];
                 const int64_t t0 = (int64_t)item.i * kBM;
                 const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
-                const int64_t kvrow = q.kv0 * H_kv + (int64_t)(item.hq / G) * q.cap;
-                if (it > 0 && !wait_bar(&bar[kQEmpty], (uint32_t)((it - 1) & 1), abort, err)) break;
-                mbar_arrive_expect_tx(&bar[kQFull], kTileBytes);
-                tma_3d(sQ, &tm_q, 0, item.hq, (int)(q.q0 + t0), &bar[kQFull]);
-                tma_3d(sQ + kHalf, &tm_q, 64, item.hq, (int)(q.q0 + t0), &bar[kQFull]);
-                ++it;
-                bool stop = false;
-                for (int j = 0; j < n_kt; j++, g++) {
-                    const int s = (int)(g & 1);
-                    const uint32_t ph = (uint32_t)(((g >> 1) - 1) & 1);
-                    // keys are free once their Q K^T is done, values once their P V is
-                    if (g >= kStages && !wait_bar(&bar[kKEmpty + s], ph, abort, err)) {
+                const int64_t kvrow = q.kv0 * H_kv + (int64_t)(item.hq0 / G) * q.cap;
+                for (int x = 0; x < item.n && !stop; x++) {
+                    // slot x's query buffer is free once its last Q K^T is done
+                    if (uq[x] > 0 &&
+                        !wait_bar(&bar[kQEmpty + x], (uint32_t)((uq[x] - 1) & 1), abort, err)) {
                         stop = true;
                         break;
                     }
+                    unsigned char *sQx = sQ + x * kTileBytes;
+                    mbar_arrive_expect_tx(&bar[kQFull + x], kTileBytes);
+                    tma_3d(sQx, &tm_q, 0, item.hq0 + x, (int)(q.q0 + t0), &bar[kQFull + x]);
+                    tma_3d(sQx + kHalf, &tm_q, 64, item.hq0 + x, (int)(q.q0 + t0), &bar[kQFull + x]);
+                    ++uq[x];
+                }
+                for (int j = 0; j < n_kt && !stop; j++) {
+                    // keys are free once their Q K^T is done, values once their P V is
                     const int y = (int)(kvrow + (int64_t)j * kBN);
+                    const int s = (int)(gk % kKStages);
+                    const int64_t u = gk / kKStages;
+                    if (gk >= kKStages &&
+                        !wait_bar(&bar[kKEmpty + s], (uint32_t)((u - 1) & 1), abort, err)) {
+                        stop = true;
+                        break;
+                    }
                     mbar_arrive_expect_tx(&bar[kKFull + s], kTileBytes);
                     tma_2d(sK + s * kTileBytes, &tm_k, 0, y, &bar[kKFull + s]);
                     tma_2d(sK + s * kTileBytes + kHalf, &tm_k, 64, y, &bar[kKFull + s]);
-                    if (g >= kStages && !wait_bar(&bar[kVEmpty + s], ph, abort, err)) {
-                        k_only = true;  // this tile's keys are in flight, its values not
+                    ++gk;
+                    if (pend_y >= 0 && !issue_v(pend_y)) {
                         stop = true;
                         break;
                     }
-                    mbar_arrive_expect_tx(&bar[kVFull + s], kTileBytes);
-                    tma_2d(sV + s * kTileBytes, &tm_v, 0, y, &bar[kVFull + s]);
-                    tma_2d(sV + s * kTileBytes + kHalf, &tm_v, 64, y, &bar[kVFull + s]);
+                    pend_y = y;
                 }
-                if (stop) break;
+                // the item's last value tile now, not behind the next item's
+                // query-buffer wait (its P V would stall on the load)
+                if (!stop && pend_y >= 0) stop = !issue_v(pend_y);
+                pend_y = -1;
             }
             // let every copy issued land before the CTA may exit
-            if (it > 0) mbar_wait_bounded(&bar[kQFull], (uint32_t)((it - 1) & 1), err);
-            for (int64_t x = g - kStages; x < g; x++) {
-                if (x < 0) continue;
-                const int s = (int)(x & 1);
-                mbar_wait_bounded(&bar[kKFull + s], (uint32_t)((x >> 1) & 1), err);
-                mbar_wait_bounded(&bar[kVFull + s], (uint32_t)((x >> 1) & 1), err);
-            }
-            if (k_only) mbar_wait_bounded(&bar[kKFull + (g & 1)], (uint32_t)((g >> 1) & 1), err);
+            for (int x = 0; x < kSlots; x++)
+                if (uq[x] > 0)
+                    mbar_wait_bounded(&bar[kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
+            for (int64_t x = gk - kKStages; x < gk; x++)
+                if (x >= 0)
+                    mbar_wait_bounded(&bar[kKFull + (int)(x % kKStages)], (uint32_t)((x / kKStages) & 1),
+                                      err);
+            for (int64_t x = gv - kVStages; x < gv; x++)
+                if (x >= 0)
+                    mbar_wait_bounded(&bar[kVFull + (int)(x % kVStages)], (uint32_t)((x / kVStages) & 1),
+                                      err);
         }
     } else if (warp == 1) {
         // ===================== MMA issue =====================
+        // Per key/value tile j of an item, for each slot x in turn:
+        //   O_x += P_x V (j), then S_x = Q_x K^T (j + 1).
+        // P_x lives in the first half of S_x's columns, so slot x's next
+        // Q K^T waits for its P V to complete; the other slot's products keep
+        // the tensor pipe busy meanwhile, and each slot's softmax overlaps
+        // the other slot's products.
         if (lane == 0) {
             const uint32_t id_qk = instr_desc(false), id_pv = instr_desc(true);
             const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV);
-            const uint32_t tS = tmem, tO = tmem + kBN, tP = tmem + 2 * kBN;
             // Descriptors are built once per buffer; a K step or a stage only
             // moves the start address, whose field (address / 16, 14 bits)
             // cannot carry over inside shared memory.
             const uint64_t dQ = smem_desc(aQ, 16, 1024);
             const uint64_t dK = smem_desc(aK, 16, 1024), dV = smem_desc(aV, kHalf, 1024);
             constexpr uint64_t kStageD = kTileBytes >> 4;
-            int64_t it = 0, g = 0;
-            bool issued = false;
-            auto pv = [&](int64_t gp, bool first_of_item) -> bool {
-                const int s = (int)(gp & 1);
-                if (!wait_bar(&bar[kPFull + s], (uint32_t)((gp >> 1) & 1), abort, err)) return false;
-                if (!wait_bar(&bar[kVFull + s], (uint32_t)((gp >> 1) & 1), abort, err)) return false;
+            int64_t g = 0;                       // key/value tiles
+            int64_t ut[kSlots] = {}, uq[kSlots] = {};  // per slot: tiles (P V issued), items
+            bool issued = false, stop = false;
+            auto qk = [&](int x, int64_t gg) -> bool {  // S_x = Q_x K^T of key tile gg
+                const int s = (int)(gg % kKStages);
+                if (x == 0 && !wait_bar(&bar[kKFull + s], (uint32_t)((gg / kKStages) & 1), abort, err))
+                    return false;
+                // P V of slot x's previous tile has read P_x (inside S_x)
+                if (ut[x] > 0 && !wait_bar(&bar[kODone + x], (uint32_t)((ut[x] - 1) & 1), abort, err))
+                    return false;
                 tc_fence_after();
-                const uint64_t dVs = dV + (uint64_t)s * kStageD;
+                const uint64_t dQx = dQ + (uint64_t)x * kStageD, dKs = dK + (uint64_t)s * kStageD;
 #pragma unroll
-                for (int kk = 0; kk < kBN / 16; kk++) {
-                    const uint64_t vo = (uint64_t)((kk * 16 * 128) >> 4);  // 16 keys further
-                    umma_tmem_a(tO, tP + s * (kBN / 2) + kk * 8, dVs + vo, id_pv,
-                                (first_of_item && kk == 0) ? 0u : 1u);
+                for (int kk = 0; kk < kD / 16; kk++) {
+                    const uint64_t ko = (uint64_t)(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
+                    umma(tmem + x * kBN, dQx + ko, dKs + ko, id_qk, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(&bar[kPFree + s]);
-                umma_commit(&bar[kVEmpty + s]);
+                umma_commit(&bar[kSFull + x]);
                 issued = true;
                 return true;
             };
-            for (int64_t k = blockIdx.x; k < total && !*abort; k += gridDim.x) {
-                const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
+            for (int64_t k = blockIdx.x; k < total && !stop && !*abort; k += gridDim.x) {
+                Req q;
+                const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
                 if (!item.valid) continue;
-                const Req &q = tab[item.b];
+                const int n = item.n;
                 const int64_t t0 = (int64_t)item.i * kBM;
                 const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
-                if (!wait_bar(&bar[kQFull], (uint32_t)(it & 1), abort, err)) break;
-                bool stop = false;
-                for (int j = 0; j < n_kt; j++, g++) {
-                    const int s = (int)(g & 1);
-                    if (!wait_bar(&bar[kKFull + s], (uint32_t)((g >> 1) & 1), abort, err) ||
-                        (g > 0 && !wait_bar(&bar[kSFree], (uint32_t)((g - 1) & 1), abort, err))) {
-                        stop = true;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint64_t dKs = dK + (uint64_t)s * kStageD;
+                for (int x = 0; x < n && !stop; x++)
+                    stop = !wait_bar(&bar[kQFull + x], (uint32_t)(uq[x] & 1), abort, err);
+                for (int x = 0; x < n && !stop; x++) stop = !qk(x, g);
+                if (stop) break;
+                umma_commit(&bar[kKEmpty + (int)(g % kKStages)]);
+                if (n_kt == 1)
+                    for (int x = 0; x < n; x++) umma_commit(&bar[kQEmpty + x]);
+                for (int j = 0; j < n_kt && !stop; j++, g++) {
+                    const int sv = (int)(g % kVStages);
+                    for (int x = 0; x < n; x++) {
+                        if (!wait_bar(&bar[kPFull + x], (uint32_t)(ut[x] & 1), abort, err) ||
+                            (x == 0 &&
+                             !wait_bar(&bar[kVFull + sv], (uint32_t)((g / kVStages) & 1), abort, err))) {
+                            stop = true;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t dVs = dV + (uint64_t)sv * kStageD;
 #pragma unroll
-                    for (int kk = 0; kk < kD / 16; kk++) {
-                        const uint64_t ko = (uint64_t)(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
-                        umma(tS, dQ + ko, dKs + ko, id_qk, kk > 0 ? 1u : 0u);
-                    }
-                    umma_commit(&bar[kSFull]);
-                    umma_commit(&bar[kKEmpty + s]);
-                    // the query tile is free once the item's last Q K^T is done
-                    if (j == n_kt - 1) umma_commit(&bar[kQEmpty]);
-                    issued = true;
-                    if (j > 0 && !pv(g - 1, j == 1)) {
-                        stop = true;
-                        break;
+                        for (int kk = 0; kk < kBN / 16; kk++) {
+                            const uint64_t vo = (uint64_t)((kk * 16 * 128) >> 4);  // 16 keys further
+                            umma_tmem_a(tmem + 2 * kBN + x * kBN, tmem + x * kBN + kk * 8, dVs + vo,
+                                        id_pv, (j == 0 && kk == 0) ? 0u : 1u);
+                        }
+                        umma_commit(&bar[kODone + x]);
+                        ++ut[x];
+                        if (x == n - 1) umma_commit(&bar[kVEmpty + sv]);  // values of tile j are read
+                        if (j + 1 < n_kt) {
+                            if (!qk(x, g + 1)) {
+                                stop = true;
+                                break;
+                            }
+                            if (x == n - 1) {
+                                umma_commit(&bar[kKEmpty + (int)((g + 1) % kKStages)]);
+                                // the query tiles are free once the item's last Q K^T is done
+                                if (j + 2 == n_kt)
+                                    for (int y = 0; y < n; y++) umma_commit(&bar[kQEmpty + y]);
+                            }
+                        }
                     }
                 }
-                if (stop || !pv(g - 1, n_kt == 1)) break;
-                ++it;
+                for (int x = 0; x < n; x++) ++uq[x];
             }
             if (issued) {  // every MMA issued has completed before TMEM is freed
                 umma_commit(&bar[kDrain]);
@@ -412,27 +501,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
     } else {
-        // ===================== softmax: one query row per thread ==========
+        // ===================== softmax: a warpgroup per slot ==========
+        const int x = (warp - 2) >> 2;        // slot
         const int quarter = warp & 3;         // TMEM lanes 32*quarter .. +31
         const int r = quarter * 32 + lane;    // the row of the tile
         const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
-        const uint32_t tS = tmem + lanes, tO = tmem + lanes + kBN, tP = tmem + lanes + 2 * kBN;
-        int64_t g = 0;
+        const uint32_t tS = tmem + lanes + x * kBN, tO = tmem + lanes + 2 * kBN + x * kBN;
+        int64_t ut = 0, g = 0;  // this slot's tiles; key/value tiles of the CTA
         bool stop = false;
         for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
-            const Item item = item_at(k, tiles_max, B, H_q, H_kv, tab);
+            Req q;
+            const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
             if (!item.valid) continue;
-            const Req &q = tab[item.b];
             const int64_t t0 = (int64_t)item.i * kBM;
             const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
             const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
+            if (x >= item.n) {  // this slot idles for the item
+                g += n_kt;
+                continue;
+            }
             const int n_full = (int)((pi_of(q, t0, w) + 1) / kBN);  // tiles no row masks
             const int64_t c = (int64_t)q.P + q.n + q.N;
             const int64_t t = t0 + r;
             const int64_t lim = pi_of(q, t < q.S ? t : (int64_t)q.S - 1, w);
             float m = -INFINITY, l = 0.f;
-            for (int j = 0; j < n_kt; j++, g++) {
-                if (!__all_sync(0xffffffffu, wait_bar(&bar[kSFull], (uint32_t)(g & 1), abort, err))) {
+            for (int j = 0; j < n_kt; j++, g++, ut++) {
+                if (!__all_sync(0xffffffffu, wait_bar(&bar[kSFull + x], (uint32_t)(ut & 1), abort, err))) {
                     stop = true;
                     break;
                 }
@@ -445,17 +539,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int vis = masked ? (int)vis64 : kBN - 1;
                 uint32_t v[128];
                 tmem_ld128(tS, v);
-                tc_fence_before();
-                mbar_arrive(&bar[kSFree]);  // S is in registers: the next Q K^T may overwrite it
-                float mx = -INFINITY;
                 if (masked) {
+                    // keys past this row's last visible one weigh 0 (scale > 0)
 #pragma unroll
                     for (int i = 0; i < kBN; i++)
-                        mx = fmaxf(mx, i <= vis ? __uint_as_float(v[i]) : -INFINITY);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < kBN; i++) mx = fmaxf(mx, __uint_as_float(v[i]));
+                        if (i > vis) v[i] = __float_as_uint(-INFINITY);
                 }
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                for (int i = 0; i < kBN; i++) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(v[i]));
+                float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
                 mx *= sl2;
                 // Lazy rescaling: the weights keep using the running maximum
                 // unless the tile's exceeds it by more than 8 (weights then
@@ -463,42 +556,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool bump = mx > m + 8.f;  // always on the first tile (m = -inf)
                 const float mu = bump ? mx : m;
                 const float corr = fast_exp2(m - mu);  // 1 without a bump, 0 on the first tile
-                float rowsum = 0.f;
+                float sums[4] = {0.f, 0.f, 0.f, 0.f};
                 uint32_t pk[64];
 #pragma unroll
                 for (int i = 0; i < kBN; i += 2) {
-                    float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mu));
-                    float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mu));
-                    if (masked) {
-                        p0 = i <= vis ? p0 : 0.f;
-                        p1 = i + 1 <= vis ? p1 : 0.f;
-                    }
-                    rowsum += p0 + p1;
+                    const float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mu));
+                    const float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mu));
+                    sums[(i >> 1) & 3] += p0 + p1;
                     __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
                     pk[i / 2] = *reinterpret_cast<uint32_t *>(&h);
                 }
-                // P of this tile goes to TMEM buffer g & 1, free once the P V
-                // of tile g - 2 is done
-                const int pb = (int)(g & 1);
-                if (g >= 2 && !__all_sync(0xffffffffu,
-                                          wait_bar(&bar[kPFree + pb], (uint32_t)(((g >> 1) - 1) & 1),
-                                                   abort, err))) {
-                    stop = true;
-                    break;
-                }
-                tc_fence_after();
-                tmem_st64(tP + pb * (kBN / 2), pk);
+                // P over the first half of S's columns (S is in registers; the
+                // P V that read the previous P completed before this Q K^T)
+                tmem_st64(tS, pk);
                 if (j > 0 && __any_sync(0xffffffffu, bump)) {
-                    // rescale O, which holds the earlier tiles' sum once the P V of
-                    // tile g - 1 is done
-                    const int qb = (int)((g - 1) & 1);
-                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kPFree + qb],
-                                                          (uint32_t)(((g - 1) >> 1) & 1), abort,
-                                                          err))) {
-                        stop = true;
-                        break;
-                    }
-                    tc_fence_after();
+                    // rescale O (the earlier tiles' sum: their P V completed
+                    // before this tile's Q K^T was issued)
                     uint32_t o[128];
                     tmem_ld128(tO, o);
 #pragma unroll
@@ -507,50 +580,52 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_st128(tO, o);
                     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 }
-                l = l * corr + rowsum;
+                l = l * corr + ((sums[0] + sums[1]) + (sums[2] + sums[3]));
                 m = mu;
-                if (e0 + kBN > c) {
+                if (x == 0 && e0 + kBN > c) {
                     // value rows at or past the compressed length: zero them
-                    const int s = (int)(g & 1);
-                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kVFull + s], (uint32_t)((g >> 1) & 1),
-                                                          abort, err))) {
+                    // (slot 0's P V reads the stage first)
+                    const int s = (int)(g % kVStages);
+                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kVFull + s],
+                                                          (uint32_t)((g / kVStages) & 1), abort,
+                                                          err))) {
                         stop = true;
                         break;
                     }
                     if (e0 + r >= c) {
                         unsigned char *row = sV + s * kTileBytes + r * 128;
 #pragma unroll
-                        for (int x = 0; x < 8; x++) {
-                            *reinterpret_cast<uint4 *>(row + x * 16) = make_uint4(0, 0, 0, 0);
-                            *reinterpret_cast<uint4 *>(row + kHalf + x * 16) = make_uint4(0, 0, 0, 0);
+                        for (int y = 0; y < 8; y++) {
+                            *reinterpret_cast<uint4 *>(row + y * 16) = make_uint4(0, 0, 0, 0);
+                            *reinterpret_cast<uint4 *>(row + kHalf + y * 16) = make_uint4(0, 0, 0, 0);
                         }
                     }
                     fence_proxy_async_shared();  // the MMA reads these rows
                 }
                 tc_fence_before();
-                mbar_arrive(&bar[kPFull + pb]);
+                mbar_arrive(&bar[kPFull + x]);
             }
             if (stop) break;
             // epilogue: O / l once the last P V is done
-            if (!__all_sync(0xffffffffu, wait_bar(&bar[kPFree + ((g - 1) & 1)],
-                                                  (uint32_t)(((g - 1) >> 1) & 1), abort, err)))
+            if (!__all_sync(0xffffffffu, wait_bar(&bar[kODone + x], (uint32_t)((ut - 1) & 1), abort,
+                                                  err)))
                 break;
             tc_fence_after();
             const float inv = 1.f / l;
-            __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq) * kD;
+            __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq0 + x) * kD;
             uint32_t o[128];
             tmem_ld128(tO, o);
             if (t < q.S) {
 #pragma unroll
-                for (int x = 0; x < 16; x++) {
+                for (int y = 0; y < 16; y++) {
                     uint32_t wv[4];
 #pragma unroll
-                    for (int y = 0; y < 4; y++) {
-                        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(o[8 * x + 2 * y]) * inv,
-                                                                 __uint_as_float(o[8 * x + 2 * y + 1]) * inv);
-                        wv[y] = *reinterpret_cast<uint32_t *>(&h);
+                    for (int z = 0; z < 4; z++) {
+                        __nv_bfloat162 h = __floats2bfloat162_rn(__uint_as_float(o[8 * y + 2 * z]) * inv,
+                                                                 __uint_as_float(o[8 * y + 2 * z + 1]) * inv);
+                        wv[z] = *reinterpret_cast<uint32_t *>(&h);
                     }
-                    *reinterpret_cast<uint4 *>(dst + x * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
+                    *reinterpret_cast<uint4 *>(dst + y * 8) = make_uint4(wv[0], wv[1], wv[2], wv[3]);
                 }
             }
             tc_fence_before();
@@ -615,13 +690,13 @@ cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t strea
         if (!encode(&tk, a.k_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
         if (!encode(&tv, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
     }
-    const size_t smem = smem_bytes(a.B);
+    const size_t smem = kSmemBytes;
     static std::once_flag once;
     static cudaError_t attr_err = cudaSuccess;
     std::call_once(once, [] {
         attr_err = cudaFuncSetAttribute(prefill_attn_kernel,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)smem_bytes(SPEECHKV_MAX_BATCH));
+                                        (int)kSmemBytes);
     });
     if (attr_err != cudaSuccess) return attr_err;
     const float sl2 = a.scale * 1.4426950408889634f;
