@@ -89,8 +89,11 @@ def test_prefill_edge_lengths(oracle, P, T, N, w):
 
 
 def test_prefill_gqa_groups(oracle):
-    """Query heads per KV head 1 and 4 (the head mapping hq / group)."""
-    for H_q, H_kv in ((8, 8), (16, 4)):
+    """Query heads per KV head 1, 3 and 4 (the head mapping hq / group).  A
+    work item holds up to two query heads of one KV head: with one head per
+    KV head the second tile of every item is idle, with three the items
+    alternate between two heads and one."""
+    for H_q, H_kv in ((8, 8), (12, 4), (16, 4)):
         wl = _wl(P=[4], T=[300], N=[20], H_q=H_q, H_kv=H_kv, seed=2003)
         L, qs, out, full = _run(wl, 8)
         _check(oracle, wl, 8, L, qs, out)
