@@ -418,6 +418,19 @@ speechkv_status speechkv_decode_step_paged(
  */
 speechkv_status speechkv_check_device_error(cudaStream_t stream);
 
+/*
+ * Self-test of the failure path shared by every kernel (no argument of the
+ * paper's method is involved): launches one CTA whose single waiting thread
+ * waits, through the same bounded wait the kernels use, for an mbarrier phase
+ * that nothing completes.  After the wait limit (1 s of %globaltimer) it
+ * gives up, records SPEECHKV_ERR_TIMEOUT in the device error word and the
+ * kernel returns normally: no trap, no fault, the context stays usable.
+ * Returns SPEECHKV_OK once launched (SPEECHKV_ERR_CUDA if the launch failed);
+ * read the recorded status with speechkv_check_device_error.  Stream-ordered,
+ * asynchronous.
+ */
+speechkv_status speechkv_selftest_timeout(cudaStream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

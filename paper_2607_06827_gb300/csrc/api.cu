@@ -309,6 +309,14 @@ speechkv_status speechkv_decode_step(const void *q, const void *k_new, const voi
                          flags, stream, true);
 }
 
+speechkv_status speechkv_selftest_timeout(cudaStream_t stream) {
+    DeviceState *s = nullptr;
+    speechkv_status st = device_state(&s);
+    if (st != SPEECHKV_OK) return st;
+    return speechkv::launch_selftest_timeout(s->err, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                           : SPEECHKV_ERR_CUDA;
+}
+
 speechkv_status speechkv_check_device_error(cudaStream_t stream) {
     DeviceState *s = nullptr;
     speechkv_status st = device_state(&s);

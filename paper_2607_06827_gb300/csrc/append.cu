@@ -51,7 +51,25 @@ __global__ void __launch_bounds__(256)
     if (threadIdx.x == 0) len[b] = (int32_t)(L + 1);
 }
 
+// One thread waits, through the bounded wait every kernel of the library
+// uses, for a phase of an mbarrier that no thread ever completes: the wait
+// gives up after its time limit, records SPEECHKV_ERR_TIMEOUT and the kernel
+// returns normally.
+__global__ void selftest_timeout_kernel(int *err) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        fence_mbar_init();
+        mbar_wait_bounded(&bar, 0, err);  // phase 0 needs one arrival: none comes
+    }
+}
+
 }  // namespace
+
+cudaError_t launch_selftest_timeout(int *err, cudaStream_t stream) {
+    selftest_timeout_kernel<<<1, 32, 0, stream>>>(err);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream) {
     if (a.dtype == SPEECHKV_F32)

@@ -67,6 +67,8 @@ struct AppendArgs {
     CacheMap map;  // paged layout when map.table != nullptr (cache_off unused)
 };
 cudaError_t launch_append(const AppendArgs &a, cudaStream_t stream);
+// A bounded wait that runs out (see speechkv_selftest_timeout).
+cudaError_t launch_selftest_timeout(int *err, cudaStream_t stream);
 
 struct DecodeArgs {
     const void *q;

@@ -61,6 +61,7 @@ SIGNATURES = {
                                              _I32, _I32, _I32, _I32, _I32, _I32, _I32,
                                              ctypes.c_int, _P]),
     "speechkv_check_device_error": (ctypes.c_int, [_P]),
+    "speechkv_selftest_timeout": (ctypes.c_int, [_P]),
 }
 
 _lock = threading.Lock()
@@ -289,3 +290,8 @@ def prefill_attn(q, q_off, P, T, N, k_cache, v_cache, cache_off, out, w: int, la
 def check_device_error(stream=None) -> int:
     """Synchronise the stream and return (and clear) the device error status."""
     return load().speechkv_check_device_error(_stream(stream))
+
+
+def selftest_timeout(stream=None):
+    """Launch the bounded-wait self-test (it records ERR_TIMEOUT after ~1 s)."""
+    _check(load().speechkv_selftest_timeout(_stream(stream)), "speechkv_selftest_timeout")
