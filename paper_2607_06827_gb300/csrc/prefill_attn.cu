@@ -678,14 +678,17 @@ cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t strea
         if (!encode(&tv, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
     }
     const size_t smem = kSmemBytes;
-    static std::once_flag once;
-    static cudaError_t attr_err = cudaSuccess;
-    std::call_once(once, [] {
-        attr_err = cudaFuncSetAttribute(prefill_attn_kernel,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        (int)kSmemBytes);
-    });
-    if (attr_err != cudaSuccess) return attr_err;
+    // the shared-memory opt-in is per device: set it once on each
+    static int configured_device_mask = 0;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (!(dev < 31 && (__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev)))) {
+        e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kSmemBytes);
+        if (e != cudaSuccess) return e;
+        if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
+    }
     const float sl2 = a.scale * 1.4426950408889634f;
     prefill_attn_kernel<<<num_sms, kThreads, smem, stream>>>(
         tq, tk, tv, a.q_off, a.P, a.T, a.N, a.cache_off, static_cast<__nv_bfloat16 *>(a.out),
