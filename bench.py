@@ -48,6 +48,8 @@ HEADLINE_MINUTES, HEADLINE_W, GENERATED = 20, 4, 64
 SWEEP = [(2, 4), (2, 8), (5, 4), (5, 8), (10, 4), (10, 8), (20, 8)]
 FALLBACK_HBM_GBS = 6800.0
 FALLBACK_BF16_TFLOPS = 1900.0
+ISOLATED_REPS = 8  # isolated single-layer replays per layer kind
+L2_FLUSH_BYTES = 256 << 20  # read before each isolated launch (L2 is 129 MB)
 POOL_BATCH = 5  # back-to-back speechkv_pool launches per timed group (setup of each layer)
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "decode_attn_traffic.txt")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_06827_gb300", "csrc", f)
@@ -348,7 +350,8 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
     layers only; (C) the full-resolution layers only -- per-layer times of
     the two kinds.  Returns a result dict."""
     import torch
-    model = DecodeModel(wl, steps_total=warmup + 3 * steps, seed_key=seed_key, layers=layers)
+    model = DecodeModel(wl, steps_total=warmup + 3 * steps + 2 * ISOLATED_REPS, seed_key=seed_key,
+                        layers=layers)
     L = len(model.layers)
     comp = [i for i, layer in enumerate(model.layers) if layer >= wl.l0]
     full = [i for i, layer in enumerate(model.layers) if layer < wl.l0]
@@ -367,6 +370,32 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
                               nb / (steps * len(pos)))
         else:
             per_kind[kind] = (float("nan"),) * 3
+    # one layer's step alone, eager, L2 flushed before each launch
+    isolated = {}
+    # the flush reads a buffer larger than L2 (a write would leave L2 full of
+    # dirty lines whose write-back would then share the HBM with the kernel)
+    flush = torch.zeros(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    for kind, pos in (("compressed", comp), ("full", full)):
+        if not pos:
+            isolated[kind] = float("nan")
+            continue
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            model.launch_step([pos[0]], fused=fused)
+        times = []
+        for _ in range(ISOLATED_REPS):
+            # the flush (tens of µs on the GPU) is still running when the
+            # events and the replay are queued, so no host latency is timed
+            flush.sum()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        del g
+        isolated[kind] = sorted(times)[len(times) // 2] * 1e3
+    del flush
     status = model.sk.check_device_error()
     assert status == model.sk.OK, model.sk.status_string(status)
     res = {
@@ -382,6 +411,11 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
         "attn_bytes_per_launch_compressed": per_kind["compressed"][2],
         "attn_us_full_layer": per_kind["full"][0],
         "attn_gbs_full_layer": per_kind["full"][1],
+        "isolated_us_compressed_layer": isolated["compressed"],
+        "isolated_us_full_layer": isolated["full"],
+        "isolated_note": (f"one layer's step alone (a one-launch CUDA graph) after reading "
+                          f"{L2_FLUSH_BYTES >> 20} MB (L2 flush), CUDA events around the replay, "
+                          f"median of {ISOLATED_REPS}"),
         "pool_us_compressed_layer": (sum(model.pool_ms[model.layers[i]] for i in comp) /
                                      len(comp) * 1e3 if comp else float("nan")),
         "pool_us_full_layer": (sum(model.pool_ms[model.layers[i]] for i in full) /
