@@ -187,3 +187,37 @@ def test_prefill_full_size_sampled(oracle):
             ref = oracle.decode_attn_request(qt, K[:last + 1], V[:last + 1],
                                              storage=oracle.STORE_BF16)
             H.assert_close(H.f64(out[off[b] + t]), ref, "bf16", f"request {b} row {t}")
+
+
+def test_prefill_random_shapes(oracle):
+    """Seeded random batches: 1-6 requests with random text and speech
+    lengths, windows 1-8, several query/KV head ratios, pooled and
+    full-resolution layers; every request against the oracle on the GPU's
+    cache, and three launches bit-identical."""
+    H.require_gpu()
+    sk = H.lib()
+    rng = np.random.default_rng(2007)
+    heads = [(2, 2), (6, 2), (8, 8), (12, 4), (16, 8)]
+    for case in range(12):
+        B = int(rng.integers(1, 7))
+        H_q, H_kv = heads[int(rng.integers(len(heads)))]
+        w = int(rng.choice([1, 2, 3, 4, 5, 8]))
+        P = [int(x) for x in rng.integers(0, 40, B)]
+        T = [int(x) for x in rng.integers(0, 500, B)]
+        N = [max(int(x), 1 if p + t == 0 else 0) for x, p, t in zip(rng.integers(0, 80, B), P, T)]
+        layer = int(rng.choice([0, 8]))
+        wl = _wl(P, T, N, w=w, seed=2100 + case, H_q=H_q, H_kv=H_kv)
+        L, full = H.gpu_prefill(wl, layer, extra_rows=int(rng.integers(0, 4)))
+        qs = [inputs.prefill_q(wl, layer, b) for b in range(wl.B)]
+        q = torch.cat(qs).cuda()
+        Pd, Td, Nd = H.lengths_dev(wl)
+        q_off = torch.from_numpy(_q_off(wl)).cuda()
+        outs = []
+        for _ in range(3):
+            out = torch.full_like(q, 3.0)
+            sk.prefill_attn(q, q_off, Pd, Td, Nd, L.k, L.v, L.cache_off, out, w, layer, wl.l0,
+                            H_kv)
+            assert sk.check_device_error() == sk.OK
+            outs.append(out)
+        assert all(torch.equal(outs[0], o) for o in outs[1:]), f"case {case}: not deterministic"
+        _check(oracle, wl, layer, L, qs, outs[0])
