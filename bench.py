@@ -443,7 +443,10 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
     its q/k/v (all layers, one copy per tensor) from pinned host memory, runs
     the layers' fused decode steps back to back (consecutive layers may
     overlap, as in the device-resident passes) and reads the outputs of all
-    layers back in one copy."""
+    layers back in one copy.  The copies run on a second stream into double
+    buffers, as a serving loop would: step s + 1's inputs come in and step
+    s's outputs go out while step s computes; every copy is inside the timed
+    region."""
     import torch
     model = DecodeModel(wl, steps_total=warmup + steps, seed_key=seed_key, layers=layers)
     L, B, Hq, Hk, d = len(model.layers), wl.B, wl.H_q, wl.H_kv, wl.d
@@ -452,25 +455,56 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
     h_kn = model.kn.cpu().pin_memory()
     h_vn = model.vn.cpu().pin_memory()
     h_out = torch.empty((total, L, B, Hq, d), dtype=model.dtype).pin_memory()
-    d_q = torch.empty((L, B, Hq, d), dtype=model.dtype, device="cuda")
-    d_kn = torch.empty((L, B, Hk, d), dtype=model.dtype, device="cuda")
-    d_vn = torch.empty((L, B, Hk, d), dtype=model.dtype, device="cuda")
+    mk = lambda *shape: torch.empty(shape, dtype=model.dtype, device="cuda")  # noqa: E731
+    d_in = [(mk(L, B, Hq, d), mk(L, B, Hk, d), mk(L, B, Hk, d)) for _ in range(2)]
+    d_out = [mk(L, B, Hq, d) for _ in range(2)]
     sk = model.sk
+    copy = torch.cuda.Stream()
 
-    def step(s):
-        d_q.copy_(h_q[s], non_blocking=True)
-        d_kn.copy_(h_kn[s], non_blocking=True)
-        d_vn.copy_(h_vn[s], non_blocking=True)
-        for i, layer in enumerate(model.layers):
-            # after the first layer the previous kernel is another layer's
-            # decode step, which writes none of this layer's cache or length
-            sk.decode_step(d_q[i], d_kn[i], d_vn[i], model.k[i], model.v[i], model.off[i],
-                           model.len[i], model.out[i], model.ws, wl.w, layer, wl.l0,
-                           flags=sk.OVERLAP_PRIOR if i > 0 else 0)
-        h_out[s].copy_(model.out, non_blocking=True)
+    def enqueue(s0, n):
+        """Steps s0 .. s0 + n - 1 on the current (compute) stream, their
+        copies on the copy stream; ends with the compute stream waiting for
+        every copy (under graph capture the current stream is the capturing
+        one, and the copy stream forks from and joins it)."""
+        comp = torch.cuda.current_stream()
+        ev_in = [torch.cuda.Event() for _ in range(n)]
+        ev_done = [torch.cuda.Event() for _ in range(n)]
+        ev_out = [torch.cuda.Event() for _ in range(n)]
+        copy.wait_stream(comp)
 
-    for s in range(warmup):
-        step(s)
+        def h2d(i):
+            q, kn, vn = d_in[i % 2]
+            with torch.cuda.stream(copy):
+                if i >= 2:
+                    copy.wait_event(ev_done[i - 2])  # step i - 2 has read this buffer
+                q.copy_(h_q[s0 + i], non_blocking=True)
+                kn.copy_(h_kn[s0 + i], non_blocking=True)
+                vn.copy_(h_vn[s0 + i], non_blocking=True)
+                ev_in[i].record(copy)
+
+        h2d(0)
+        for i in range(n):
+            if i + 1 < n:
+                h2d(i + 1)
+            q, kn, vn = d_in[i % 2]
+            out = d_out[i % 2]
+            comp.wait_event(ev_in[i])
+            if i >= 2:
+                comp.wait_event(ev_out[i - 2])  # step i - 2's outputs have left
+            for j, layer in enumerate(model.layers):
+                # after the first layer the previous kernel is another layer's
+                # decode step, which writes none of this layer's cache or length
+                sk.decode_step(q[j], kn[j], vn[j], model.k[j], model.v[j], model.off[j],
+                               model.len[j], out[j], model.ws, wl.w, layer, wl.l0,
+                               flags=sk.OVERLAP_PRIOR if j > 0 else 0)
+            ev_done[i].record(comp)
+            with torch.cuda.stream(copy):
+                copy.wait_event(ev_done[i])
+                h_out[s0 + i].copy_(out, non_blocking=True)
+                ev_out[i].record(copy)
+        comp.wait_stream(copy)
+
+    enqueue(0, warmup)
     torch.cuda.synchronize()
     graphs = []
     s = warmup
@@ -478,8 +512,7 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
         n = min(chunk, total - s)
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            for i in range(n):
-                step(s + i)
+            enqueue(s, n)
         graphs.append(g)
         s += n
     dist.barrier()
@@ -497,13 +530,14 @@ def measure_e2e(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, see
     assert status == sk.OK, sk.status_string(status)
     ok = bool(torch.isfinite(h_out[warmup:].float()).all())
     esz = 2
-    h2d = L * B * (Hq + 2 * Hk) * d * esz
-    d2h = L * B * Hq * d * esz
+    h2d_bytes = L * B * (Hq + 2 * Hk) * d * esz
+    d2h_bytes = L * B * Hq * d * esz
     del graphs
     model.free()
     torch.cuda.empty_cache()
-    return {"value": region_ms * 1e3 / steps / L, "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": d2h, "steps": steps, "outputs_finite": ok}
+    return {"value": region_ms * 1e3 / steps / L, "unit": UNIT, "h2d_bytes_per_step": h2d_bytes,
+            "d2h_bytes_per_step": d2h_bytes, "steps": steps, "outputs_finite": ok,
+            "copies": "second stream, double-buffered, overlapping the neighbouring steps"}
 
 
 def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
