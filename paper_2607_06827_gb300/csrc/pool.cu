@@ -570,7 +570,10 @@ inline HsPlan hs_plan(int VR) {
     // two vectors per lane up to 4 KB rows (teams of up to four warps, up
     // to 16 warps per CTA), four for wider rows (registers: 12 warps)
     p.vpl = VR <= 32 ? 1 : VR <= 256 ? 2 : 4;
-    p.g = (VR + 32 * p.vpl - 1) / (32 * p.vpl);
+    // warps per team, rounded up to a compiled team size (1, 2, 4 or 8); the
+    // lanes past the row's last vector idle
+    const int g = (VR + 32 * p.vpl - 1) / (32 * p.vpl);
+    p.g = g <= 1 ? 1 : g <= 2 ? 2 : g <= 4 ? 4 : 8;
     const int max_warps = p.vpl >= 4 ? 12 : kHsMaxWarps;
     const int64_t stage = (int64_t)kPoolFrames * VR * 16;
     const int slots = (int)(kHsRingBytes / stage);  // >= 3 for rows of up to 16 KB
@@ -615,6 +618,8 @@ cudaError_t launch_pool_hidden_instance(const PoolHiddenArgs &a, int num_sms,
                                         cudaStream_t stream) {
     const int VR = (int)((int64_t)a.d_model * (int64_t)sizeof(T) / 16);
     const HsPlan p = hs_plan(VR);
+    // (vpl, g): (1, 1) rows of up to 32 vectors; (2, 1 / 2 / 4) up to 256;
+    // (4, 4 / 8) up to 1024 -- a team covers 32 * vpl * g >= VR vectors
     if (p.vpl == 4)
         return p.g == 8 ? launch_pool_hidden_cfg<T, 4, 8>(a, p, num_sms, VR, stream)
                         : launch_pool_hidden_cfg<T, 4, 4>(a, p, num_sms, VR, stream);

@@ -70,20 +70,23 @@ def test_hs_pool_bf16_qwen_width(oracle, w):
     _check(oracle, wl, 2048, hs, gate, out, out_off, ln)
 
 
-@pytest.mark.parametrize("d_model", [512, 4096])
+@pytest.mark.parametrize("d_model", [512, 768, 4096])
 def test_hs_pool_fp32(oracle, d_model):
-    """fp32 storage (tolerance 1e-5), one and four vectors per thread."""
+    """fp32 storage (tolerance 1e-5), two and four vectors per lane (768:
+    a team of three warps rounded up to four)."""
     wl = _wl(dtype="f32", P=(3, 0), T=(77, 9), N=(2, 5), w=4, seed=3002)
     sk, hs, gate, out, out_off, ln = _run(wl, d_model)
     assert sk.check_device_error() == sk.OK
     _check(oracle, wl, d_model, hs, gate, out, out_off, ln)
 
 
-@pytest.mark.parametrize("d_model,w", [(256, 4), (512, 3), (1024, 4), (4096, 4), (8192, 5)])
+@pytest.mark.parametrize("d_model,w", [(256, 4), (512, 3), (1024, 4), (1536, 4), (2560, 3),
+                                       (4096, 4), (5120, 4), (8192, 5)])
 def test_hs_pool_bf16_row_widths(oracle, d_model, w):
     """Rows of 0.5 to 16 KB (one to four vectors per lane, teams of one to
-    eight warps); w = 5 splits every window into a full group of frames and
-    a ragged one."""
+    eight warps), including widths whose team is rounded up to the next
+    compiled size (1536: 3 -> 4 warps; 2560: 3 -> 4; 5120: 5 -> 8); w = 5
+    splits every window into a full group of frames and a ragged one."""
     wl = _wl(P=(2, 0), T=(151, 64), N=(3, 9), w=w, seed=3005)
     sk, hs, gate, out, out_off, ln = _run(wl, d_model)
     assert sk.check_device_error() == sk.OK
