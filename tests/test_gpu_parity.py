@@ -67,6 +67,8 @@ POOL_CASES = [
     ("bf16", 64, 4, (0, 5), (40, 41), (8, 0), 8),
     ("f32", 128, 2, (0,), (50,), (6,), 2),
     ("bf16", 128, 8, (0,), (17,), (2,), 1),           # w = 1: bit-exact copy
+    ("bf16", 128, 3, (0, 2), (90, 37), (5, 0), 4),    # odd H_kv: a half-empty warp chunk
+    ("f32", 64, 1, (1,), (20,), (2,), 3),             # one KV head
 ]
 
 
@@ -168,6 +170,8 @@ ATTN_CASES = [
     ("bf16", 128, 16, 4, (0,), (500,), (20,), (3,), 8),           # group 4
     ("bf16", 64, 8, 4, (0, 0, 4), (63, 1500, 0), (16, 256, 9), (0, 512, 3), 4),
     ("f32", 64, 16, 4, (2,), (33,), (1,), (0,), 2),
+    ("bf16", 128, 6, 3, (0, 2), (200, 50), (10, 4), (3, 0), 4),  # odd H_kv, group 2
+    ("bf16", 64, 5, 5, (0,), (120,), (6,), (1,), 4),              # H_kv = 5, group 1
 ]
 
 
