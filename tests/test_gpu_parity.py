@@ -485,3 +485,33 @@ def test_full_size_ragged_sampled(sk, oracle, fused):
 def test_full_size_long_audio_fused(sk, oracle):
     wl = inputs.qwen_long_audio(20, 4, generated=64)
     _sampled_full_size(sk, oracle, wl, wl.l0, samples=[3], fused=True)
+
+
+def test_max_batch_fused_step(sk, oracle):
+    """B = SPEECHKV_MAX_BATCH (the largest per-request tables in shared
+    memory), short random lengths: pooling, one fused decode step, sampled
+    requests against the oracle."""
+    rng = np.random.default_rng(4242)
+    B = sk.MAX_BATCH
+    T = [int(x) for x in rng.integers(1, 60, B)]
+    N = [int(x) for x in rng.integers(0, 20, B)]
+    wl = inputs.Workload(name="maxbatch", dtype="bf16", L=28, l0=8, w=4, H_q=16, H_kv=8, d=128,
+                         P=[0] * B, T=T, N=N, G=[0] * B, steps=1, seed=4242)
+    layer = wl.l0
+    L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=1)
+    ws = sk.new_workspace(wl.B, wl.H_q, wl.H_kv, wl.d)
+    q, kn, vn = inputs.step_qkv(wl, layer, 0)
+    out = torch.empty_like(q, device="cuda")
+    sk.decode_step(q.cuda(), kn.cuda(), vn.cuda(), L.k, L.v, L.cache_off, L.len, out, ws, wl.w,
+                   layer, wl.l0)
+    assert sk.check_device_error() == sk.OK
+    for b in sorted(set([0, 1, B - 1] + [int(x) for x in rng.integers(0, B, 13)])):
+        Ko, Vo = oracle.pool_request(H.f64(ks[b]), H.f64(vs[b]), 0, T[b], N[b], H.f64(gate),
+                                     wl.w, layer, wl.l0, storage=oracle.STORE_BF16)
+        n = Ko.shape[0]
+        Kc = np.zeros((n + 1, wl.H_kv, wl.d)); Vc = np.zeros_like(Kc)
+        Kc[:n], Vc[:n] = Ko, Vo
+        n = oracle.append_request(Kc, Vc, n, H.f64(kn[b]), H.f64(vn[b]))
+        assert int(L.len[b]) == n
+        ref = oracle.decode_attn_request(H.f64(q[b]), Kc[:n], Vc[:n], storage=oracle.STORE_BF16)
+        H.assert_close(H.f64(out[b]), ref, "bf16", f"request {b}")

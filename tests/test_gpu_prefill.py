@@ -221,3 +221,19 @@ def test_prefill_random_shapes(oracle):
             outs.append(out)
         assert all(torch.equal(outs[0], o) for o in outs[1:]), f"case {case}: not deterministic"
         _check(oracle, wl, layer, L, qs, outs[0])
+
+
+def test_prefill_max_batch(oracle):
+    """B = SPEECHKV_MAX_BATCH requests with short random lengths (many small
+    items, the request table read per item), every request against the
+    oracle."""
+    H.require_gpu()
+    sk = H.lib()
+    rng = np.random.default_rng(2011)
+    B = sk.MAX_BATCH
+    T = [int(x) for x in rng.integers(0, 200, B)]
+    N = [int(x) for x in rng.integers(1, 40, B)]
+    P = [int(x) for x in rng.integers(0, 8, B)]
+    wl = _wl(P, T, N, w=4, seed=2011)
+    L, qs, out, full = _run(wl, 8)
+    _check(oracle, wl, 8, L, qs, out)
