@@ -372,7 +372,10 @@ speechkv_status speechkv_decode_step_noalloc(
  *              [0, num_blocks) for every row the call reads or writes
  *              (others may hold anything, e.g. -1).
  * block_size   a power of two; each request's capacity is
- *              max_blocks * block_size rows (at most 2^31 - 1).
+ *              max_blocks * block_size rows (at most 2^31 - 1).  The
+ *              decode step reads a 128-row tile as one copy per page
+ *              segment: pages of 64 rows or more keep it within ~7 % of
+ *              the contiguous layout; 16-row pages cost up to ~1.8x.
  * num_blocks   host: pages in k_pages / v_pages (bounds the table entries).
  * The other arguments, the results and the errors are those of the
  * contiguous entry point of the same name (the rows and their order are the
