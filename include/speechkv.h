@@ -69,16 +69,20 @@ typedef enum { SPEECHKV_F32 = 0, SPEECHKV_BF16 = 1 } speechkv_dtype;
 #define SPEECHKV_MAX_BATCH 512
 
 /*
- * Flag of speechkv_decode_attn / speechkv_decode_step.  The decode kernels
- * are launched with programmatic dependent launch, so they may begin while
- * the previous kernel on the stream retires.  By default they wait for that
- * kernel before reading anything.  SPEECHKV_OVERLAP_PRIOR declares that the
- * previous kernel on `stream` writes none of this call's caches, len or
- * cache_off (it may produce q, k_new and v_new, and may use the same
- * workspace): the call then reads the lengths and starts streaming the
- * cached rows at once, and waits for the previous kernel only before
- * reading q / k_new / v_new and before any write.  A kernel that precedes
- * it without the launch attribute is simply waited for, as usual.
+ * Flag of speechkv_decode_attn / speechkv_decode_step (and their paged and
+ * allocation-free forms).  The decode kernels are launched with programmatic
+ * dependent launch, so they may begin while the previous kernel on the
+ * stream retires.  By default they wait for that kernel before reading
+ * anything.  SPEECHKV_OVERLAP_PRIOR declares that the previous kernel on
+ * `stream` writes none of this call's caches, len or cache_off (it may
+ * produce q, k_new and v_new, and may use the same workspace): the call then
+ * reads the lengths and starts streaming the cached rows at once, and waits
+ * for the previous kernel only before reading q / k_new / v_new and before
+ * any write.  Only that one kernel can still be running: a decode kernel
+ * lets its successor start only after its own wait for its predecessor has
+ * returned, so every kernel queued before the previous one has completed by
+ * then, whatever grid sizes the calls use.  A kernel that precedes the call
+ * without the launch attribute is simply waited for, as usual.
  */
 #define SPEECHKV_OVERLAP_PRIOR 1u
 
@@ -347,9 +351,13 @@ speechkv_status speechkv_decode_step(const void *q, const void *k_new,
  * SPEECHKV_ERR_WORKSPACE before anything runs.  The first call on a device
  * looks up the array's device address (a one-time set-up per device); make
  * that first call before any stream capture.  Every call shares the one
- * array, which keeps the previous call's contents: each call zeroes the
- * counters it needs on `stream` before launching, and calls that may run at
- * the same time on one device (for example on two streams) race on it.
+ * array, which keeps the previous call's contents: once all arguments have
+ * passed the host checks, each call zeroes the counters it needs on `stream`
+ * (an asynchronous memset, not an allocation) and then launches, and calls
+ * that may run at the same time on one device (for example on two streams)
+ * race on it.  Because that memset sits between the previous kernel and
+ * the decode kernel, SPEECHKV_OVERLAP_PRIOR is accepted but gives no
+ * overlap here.
  */
 #define SPEECHKV_NOALLOC_SCRATCH_BYTES (8u << 20)
 

@@ -109,15 +109,19 @@ size_t workspace_bytes(int B, int H_q, int H_kv, int d, int grid) {
     return counters_bytes(B, H_kv) + ((size_t)grid + S) * slot * 4;
 }
 
-// Shared by speechkv_decode_attn (k_new == v_new == NULL) and
-// speechkv_decode_step (both non-NULL).
-speechkv_status decode_common(const void *q, const void *k_new, const void *v_new,
-                              void *k_cache, void *v_cache, const int64_t *cache_off,
-                              int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
-                              int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
-                              int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
-                              speechkv_dtype dtype, uint32_t flags, cudaStream_t stream,
-                              bool append, const speechkv::CacheMap &map = {}) {
+// Host checks of a decode call and its launch descriptor; nothing is queued
+// on the stream.  *launch stays false when there is nothing to launch
+// (B == 0).  Shared by speechkv_decode_attn (k_new == v_new == NULL) and the
+// decode steps (both non-NULL).
+speechkv_status decode_prepare(const void *q, const void *k_new, const void *v_new,
+                               void *k_cache, void *v_cache, const int64_t *cache_off,
+                               int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+                               int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+                               int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                               speechkv_dtype dtype, uint32_t flags, bool append,
+                               const speechkv::CacheMap &map, speechkv::DecodeArgs *out_args,
+                               int *out_grid, bool *launch) {
+    *launch = false;
     if (B < 0 || H_q < 1 || H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 ||
         grid_ctas < 0 || !valid_dtype(dtype) || isnan(scale) || isinf(scale) ||
         (flags & ~SPEECHKV_OVERLAP_PRIOR))
@@ -165,6 +169,27 @@ speechkv_status decode_common(const void *q, const void *k_new, const void *v_ne
     a.err = s->err;
     a.overlap = (flags & SPEECHKV_OVERLAP_PRIOR) != 0;
     a.map = map;
+    *out_args = a;
+    *out_grid = grid;
+    *launch = true;
+    return SPEECHKV_OK;
+}
+
+speechkv_status decode_common(const void *q, const void *k_new, const void *v_new,
+                              void *k_cache, void *v_cache, const int64_t *cache_off,
+                              int32_t *len, void *out, float scale, int32_t B, int32_t H_q,
+                              int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+                              int32_t grid_ctas, void *workspace, size_t workspace_bytes_in,
+                              speechkv_dtype dtype, uint32_t flags, cudaStream_t stream,
+                              bool append, const speechkv::CacheMap &map = {}) {
+    speechkv::DecodeArgs a;
+    int grid = 0;
+    bool launch = false;
+    const speechkv_status st =
+        decode_prepare(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
+                       H_kv, d, w, layer, l0, grid_ctas, workspace, workspace_bytes_in, dtype,
+                       flags, append, map, &a, &grid, &launch);
+    if (st != SPEECHKV_OK || !launch) return st;
     return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
                                                                    : SPEECHKV_ERR_CUDA;
 }
@@ -481,12 +506,18 @@ extern "C" speechkv_status speechkv_decode_step_noalloc(
     // a batch whose scratch would not fit is refused before anything runs
     if (workspace_bytes(B, H_q, H_kv, d, grid) > (size_t)SPEECHKV_NOALLOC_SCRATCH_BYTES)
         return SPEECHKV_ERR_WORKSPACE;
+    // every other argument is checked before anything is queued on the stream
+    speechkv::DecodeArgs a;
+    bool launch = false;
+    st = decode_prepare(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
+                        H_kv, d, w, layer, l0, grid, scratch, SPEECHKV_NOALLOC_SCRATCH_BYTES,
+                        dtype, flags, true, {}, &a, &grid, &launch);
+    if (st != SPEECHKV_OK || !launch) return st;
     // the counters must start at zero; the array keeps the previous call's data
     if (cudaMemsetAsync(scratch, 0, counters_bytes(B, H_kv), stream) != cudaSuccess)
         return SPEECHKV_ERR_CUDA;
-    return decode_common(q, k_new, v_new, k_cache, v_cache, cache_off, len, out, scale, B, H_q,
-                         H_kv, d, w, layer, l0, grid, scratch, SPEECHKV_NOALLOC_SCRATCH_BYTES,
-                         dtype, flags, stream, true);
+    return speechkv::launch_decode(a, grid, stream) == cudaSuccess ? SPEECHKV_OK
+                                                                   : SPEECHKV_ERR_CUDA;
 }
 
 extern "C" speechkv_status speechkv_decode_step_paged(

@@ -4,17 +4,16 @@
 //
 // Design (GB300, HBM-bound, about 2 flop per byte):
 //   * Work = sum over requests of len[b] rows times H_kv heads.  A persistent
-//     grid (three small CTAs per SM) cuts this flat range evenly (stream-K):
-//     CTA c owns units [U*c/C, U*(c+1)/C), whatever the length mix of the
-//     batch.  Its range splits into "pieces", each a run of rows of one
-//     (request, KV head).
+//     grid (one CTA per SM: ~217 KB of shared memory each) cuts this flat
+//     range evenly (stream-K): CTA c owns units [U*c/C, U*(c+1)/C), whatever
+//     the length mix of the batch.  Its range splits into "pieces", each a
+//     run of rows of one (request, KV head).
 //   * The cache is head-major per request, so a piece is one contiguous run
-//     of rows.  One producer lane streams it HBM -> shared memory in 64-row
-//     tiles with bulk asynchronous copies (TMA, cp.async.bulk: one copy for
-//     the keys, one for the values, plus the piece's queries with its first
-//     tile) into a two-stage ring guarded by mbarriers.  Four consumer warps
-//     take 16 rows each of every tile.  Several CTAs per SM keep the memory
-//     pipe busy while one of them merges a piece.
+//     of rows.  One producer lane streams it HBM -> shared memory in tiles of
+//     128 rows (64 for 512-byte rows) with bulk asynchronous copies (TMA,
+//     cp.async.bulk: one copy for the keys, one for the values, plus the
+//     piece's queries with its first tile) into a three-stage ring guarded by
+//     mbarriers.  Eight consumer warps take 16 (8) rows each of every tile.
 //   * All G = H_q/H_kv query heads of the KV head are served from one read of
 //     each key/value row.  QK: four lanes per row, each reading a quarter of
 //     the row from shared memory in an order that keeps every 8-lane phase on
@@ -22,12 +21,13 @@
 //     online (running max and sum per warp) in base 2, with log2(e)/sqrt(d)
 //     folded into the query.  PV: each lane owns one 16-byte column chunk of
 //     a row (two rows per warp instruction for bf16, d = 128), f32x2 FMAs.
-//   * At the end of a piece the consumer warps' (max, sum, o) states are
-//     merged in shared memory.  A piece covering a whole (request, head)
-//     writes the output; otherwise it writes an unnormalised partial, and the
-//     CTA that arrives last at that (request, head) (atomic ticket with
-//     acquire-release ordering, no waiting) merges the partials with
-//     log-sum-exp weights and resets the ticket for the next call.
+//   * At the end of a piece the consumer warps deposit their (max, sum, o)
+//     states in one of two shared buffers and go on; a merge warp combines
+//     them.  A piece covering a whole (request, head) writes the output;
+//     otherwise it writes an unnormalised partial, and the CTA that arrives
+//     last at that (request, head) (atomic ticket with acquire-release
+//     ordering, no waiting) merges the partials with log-sum-exp weights and
+//     resets the ticket for the next call.
 //   * Every mbarrier wait is bounded; on timeout the kernel reports
 //     SPEECHKV_ERR_TIMEOUT, stops issuing and computing, lets its copies in
 //     flight land and returns.
@@ -154,16 +154,24 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int warp = tid >> 5, lane = tid & 31;
     const int H_q = H_kv * G;
 
-    // Programmatic dependent launch: the next kernel may start as our CTAs
-    // retire.  Unless the caller declared that the previous kernel on the
-    // stream produces at most q, k_new and v_new (overlap != 0), wait for it
-    // before touching anything.  With overlap, the prologue and the bulk
-    // copies of cached rows run first; every read of q / k_new / v_new and
-    // every global write (outputs, cache rows, len, workspace) comes after
-    // griddep_wait(), and every warp but the producer's idle lanes waits
-    // before it exits (so this grid never completes before the previous one).
-    griddep_launch_dependents();
-    if (!overlap) griddep_wait();
+    // Programmatic dependent launch.  Unless the caller declared that the
+    // previous kernel on the stream produces at most q, k_new and v_new
+    // (overlap != 0), wait for it before touching anything.  With overlap,
+    // the prologue and the bulk copies of cached rows run first; every read
+    // of q / k_new / v_new and every global write (outputs, cache rows, len,
+    // workspace) comes after griddep_wait(), and every warp but the
+    // producer's idle lanes waits before it exits (so this grid never
+    // completes before the previous one).
+    // The next kernel is released (griddep_release) only after this thread's
+    // own wait has returned, i.e. once the previous grid has completed.  So
+    // when a grid starts, every grid before its immediate predecessor has
+    // completed, whatever the grid sizes: the reads done before the wait can
+    // only overlap the one kernel the overlap contract speaks of.
+    auto griddep_release = [&]() {
+        griddep_wait();
+        griddep_launch_dependents();
+    };
+    if (!overlap) griddep_release();
 
     // ---- 1. per-request lengths (clamped to capacity) and their prefix sums
     for (int b = tid; b < B; b += blockDim.x) {
@@ -173,7 +181,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         const int64_t o0 = map.table ? (int64_t)b * capP : cache_off[b];
         const int64_t o1 = map.table ? (int64_t)(b + 1) * capP : cache_off[b + 1];
         const int64_t cap = o1 - o0;
-        int64_t L = len[b];
+        int64_t L = __ldcg(len + b);  // at L2: another grid's CTA wrote it
         int32_t nr = -1;
         if (cap < 0 || o0 < 0) {
             if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
@@ -234,7 +242,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     // consumers only once the first tile -- whose queries are copied after
     // that wait -- has landed.
     auto merge_warp_prior_part = [&]() {  // merge warp
-        griddep_wait();
+        griddep_release();
         // empty requests get a zero output (softmax over nothing)
         for (int b = blockIdx.x; b < B; b += gridDim.x) {
             if (cum[b + 1] != cum[b]) continue;
@@ -257,7 +265,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         }
     };
     auto consumer_prior_part = [&]() {  // consumer warps
-        griddep_wait();
+        griddep_release();
         if (kAppend) {
             // write the new tokens into their cache rows (nothing in this
             // kernel reads those rows from the cache: the attention takes the
@@ -289,7 +297,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         else if (warp < W)
             consumer_prior_part();
         else
-            griddep_wait();
+            griddep_release();
         return;
     }
     const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
@@ -323,7 +331,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 deferred[ndeferred++] = Deferred{dst, src, bytes, bar};
         };
         auto flush_deferred = [&]() {
-            griddep_wait();
+            griddep_release();
             waited = true;
             for (int i = 0; i < ndeferred; i++)
                 bulk_g2s(deferred[i].dst, deferred[i].src, deferred[i].bytes, deferred[i].bar);
@@ -734,7 +742,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         u += p.t1 - p.t0;
     }
     if (!prior_part_done) consumer_prior_part();  // (only if there was no tile)
-    griddep_wait();
+    griddep_release();
 }
 
 template <typename T, int D, int G, bool kAppend>

@@ -634,14 +634,21 @@ cudaError_t launch_pool_hidden_instance(const PoolHiddenArgs &a, int num_sms,
 template <typename T, int D>
 cudaError_t launch_pool_instance(const PoolArgs &a, int num_sms, cudaStream_t stream) {
     // enough CTAs over the whole batch to fill every SM once, at least one
-    // per request
-    static int per_sm = 0;
+    // per request; the occupancy is cached per device (a racing first use
+    // stores the same value, atomically)
+    constexpr int kDevs = 64;
+    static int occ_cache[kDevs] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const bool cacheable = dev >= 0 && dev < kDevs;
+    int per_sm = cacheable ? __atomic_load_n(&occ_cache[dev], __ATOMIC_ACQUIRE) : 0;
     if (per_sm == 0) {
         int occ = 0;
-        cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, pool_kernel<T, D>,
-                                                                      kPoolThreads, 0);
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, pool_kernel<T, D>, kPoolThreads, 0);
         if (e != cudaSuccess) return e;
         per_sm = occ > 0 ? occ : 1;
+        if (cacheable) __atomic_store_n(&occ_cache[dev], per_sm, __ATOMIC_RELEASE);
     }
     int64_t x = ((int64_t)per_sm * num_sms + a.B - 1) / a.B;
     if (x < 1) x = 1;

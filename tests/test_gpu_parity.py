@@ -515,3 +515,101 @@ def test_max_batch_fused_step(sk, oracle):
         assert int(L.len[b]) == n
         ref = oracle.decode_attn_request(H.f64(q[b]), Kc[:n], Vc[:n], storage=oracle.STORE_BF16)
         H.assert_close(H.f64(out[b]), ref, "bf16", f"request {b}")
+
+
+@pytest.mark.parametrize("grid", [0, 7, 16])
+def test_overlap_prior_two_layer_interleave_any_grid(sk, oracle, grid):
+    """SPEECHKV_OVERLAP_PRIOR with the steps of two layers interleaved
+    [a, b, a, b, ...]: the kernel two launches back writes this call's cache
+    and length.  A decode kernel releases its successor only after its own
+    wait for its predecessor, so that kernel has completed before this one
+    starts, whatever the grid -- small explicit grids, under which several
+    grids fit on the GPU at once, included."""
+    wl = inputs.qwen_ragged(B=5)
+    layers, steps = [wl.l0 - 1, wl.l0], 4
+    gl, ol = [], []
+    for layer in layers:
+        L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=steps)
+        gl.append(L)
+        ol.append(H.oracle_prefill(oracle, wl, layer, steps, ks, vs, gate))
+    ws = _ws(sk, wl, grid)
+    ins = [[[x.cuda() for x in inputs.step_qkv(wl, layer, t)] for layer in layers]
+           for t in range(steps)]
+    outs = [[torch.empty_like(ins[0][0][0]) for _ in layers] for _ in range(steps)]
+    for t in range(steps):
+        for i, layer in enumerate(layers):
+            q, kn, vn = ins[t][i]
+            L = gl[i]
+            sk.decode_step(q, kn, vn, L.k, L.v, L.cache_off, L.len, outs[t][i], ws, wl.w, layer,
+                           wl.l0, grid_ctas=grid, flags=sk.OVERLAP_PRIOR)
+    torch.cuda.synchronize()
+    assert sk.check_device_error() == sk.OK
+    for t in range(steps):
+        for i, layer in enumerate(layers):
+            q, kn, vn = (x.cpu() for x in ins[t][i])
+            ref = []
+            for b in range(wl.B):
+                Kc, Vc, n = ol[i][b]
+                n = oracle.append_request(Kc, Vc, n, H.f64(kn[b]), H.f64(vn[b]))
+                ol[i][b][2] = n
+                ref.append(oracle.decode_attn_request(H.f64(q[b]), Kc[:n], Vc[:n],
+                                                      storage=oracle.STORE_BF16))
+            H.assert_close(H.f64(outs[t][i]), np.stack(ref), "bf16",
+                           f"grid {grid} step {t} layer {layer}")
+    for i in range(len(layers)):
+        assert [int(x) for x in gl[i].len.cpu()] == [o[2] for o in ol[i]]
+        # every appended row sits where the oracle put it (no row written twice)
+        for b in range(wl.B):
+            K, V = gl[i].request_rows(b)
+            Kc, Vc, n = ol[i][b]
+            np.testing.assert_array_equal(K[n - steps:], Kc[n - steps:n])
+            np.testing.assert_array_equal(V[n - steps:], Vc[n - steps:n])
+
+
+# --------------------------------------------------------------------------
+# pooling at the long-audio benchmark's full size, element by element
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("minutes,w,T", [(20, 4, None), (20, 4, 14999), (10, 8, None)])
+def test_pool_full_size_matches_oracle(sk, oracle, minutes, w, T):
+    """The pooled layer l0 of the long-audio batch (8 requests; 20 min is
+    15,000 frames, with a 14,999-frame variant whose last window holds three
+    frames), every row of every KV head of the first and the last request
+    against Eq. (pool) in the oracle.  Text rows are bit-exact copies."""
+    wl = inputs.qwen_long_audio(minutes, w)
+    if T is not None:
+        wl = dataclasses.replace(wl, T=[T] * wl.B)
+    layer = wl.l0
+    L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=1)
+    assert sk.check_device_error() == sk.OK
+    lens = L.len.cpu().numpy()
+    for b in range(wl.B):
+        assert lens[b] == oracle.compressed_len(wl.P[b], wl.T[b], wl.N[b], 0, w, layer, wl.l0)
+    for b in (0, wl.B - 1):
+        Ko, Vo = oracle.pool_request(H.f64(ks[b]), H.f64(vs[b]), wl.P[b], wl.T[b], wl.N[b],
+                                     H.f64(gate), w, layer, wl.l0, storage=oracle.STORE_BF16)
+        K, V = L.request_rows(b)
+        H.assert_close(K, Ko, "bf16", f"pooled K, request {b}")
+        H.assert_close(V, Vo, "bf16", f"pooled V, request {b}")
+        n = Ko.shape[0] - wl.P[b] - wl.N[b]
+        # the first, a middle and the last (possibly partial) window, tighter:
+        # one rounding to bf16 of the fp32 result
+        for i in (0, n // 2, n - 1):
+            np.testing.assert_allclose(K[wl.P[b] + i], Ko[wl.P[b] + i], rtol=2 ** -7, atol=1e-6)
+            np.testing.assert_allclose(V[wl.P[b] + i], Vo[wl.P[b] + i], rtol=2 ** -7, atol=1e-6)
+        src_k, src_v = H.f64(ks[b]), H.f64(vs[b])
+        np.testing.assert_array_equal(K[wl.P[b] + n:], src_k[wl.P[b] + wl.T[b]:])
+        np.testing.assert_array_equal(V[wl.P[b] + n:], src_v[wl.P[b] + wl.T[b]:])
+
+
+# --------------------------------------------------------------------------
+# batch of 64 uniform 30 s requests, compressed and uncompressed
+# --------------------------------------------------------------------------
+@pytest.mark.parametrize("w", [4, 1])
+def test_batch64_30s_pool_and_fused_steps(sk, oracle, w):
+    """64 requests of 30 s audio (375 frames) and a 32-token prompt at
+    Qwen3-1.7B shapes, pooled with w = 4 from l0 = 8 and its uncompressed
+    twin (w = 1, identical seeded tensors): pooling, then three fused decode
+    steps at layers l0 - 1 and l0, every request against the oracle's
+    pooling -> appends -> attention."""
+    wl = inputs.qwen_batch64(w=w)
+    _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=3, fused=True)
