@@ -72,14 +72,16 @@ def parse_args():
     ap.add_argument("--no-unfused", action="store_true",
                     help="skip timing append + decode_attn as two launches")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the batch-1, batch-64 and ragged-128 workloads")
     ap.add_argument("--no-paged", action="store_true",
                     help="skip the paged-cache decode measurement")
     ap.add_argument("--no-prefill", action="store_true",
                     help="skip the prefill-attention measurement")
     ap.add_argument("--prefill-only", action="store_true",
                     help="diagnostic: time only the prefill attention and print its section")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0,
-                    help="budget of the oracle CPU baseline sample")
+    ap.add_argument("--cpu-steps", type=int, default=3,
+                    help="timed whole oracle decode steps of the CPU baseline")
     ap.add_argument("--graph-chunk", type=int, default=32)
     ap.add_argument("--layers", type=str, default=None,
                     help="comma-separated layer indices to build (default: all 28); "
@@ -762,141 +764,258 @@ def measure_hs_pool(wl, clocks, repeats: int = 5, warmup: int = 2, d_model: int 
 
 
 # ---------------------------------------------------------------------------
-# CPU oracle timing (cpu_baseline and --impl reference)
+# the other workloads: batch 1 x 30 s, batch 64 x 30 s, ragged 128 requests
 # ---------------------------------------------------------------------------
-def oracle_sample_inputs(minutes: int, w: int, seed: int = 1004):
-    """One (request, KV head) of the headline workload, built by the oracle
-    itself from numpy inputs: a pooled layer (l >= l0) and a full-resolution
-    layer, each with its G generated rows.  Returns {kind: (q, K, V)}."""
+def config_workloads(w: int):
+    """The three other decode workloads at Qwen3-1.7B shapes (bf16, l0 = 8)
+    at window w, each mid-run: {name: (workload, description)}.  The ragged
+    batch's already-generated tokens are laid down at prefill as text rows
+    after the prompt (same rows and layout as appended tokens)."""
+    import dataclasses
+    from paper_2607_06827_gb300 import inputs
+    one = inputs.qwen_single()
+    one = dataclasses.replace(one, w=w, G=[one.steps // 2])
+    b64 = inputs.qwen_batch64(w=w)
+    b64 = dataclasses.replace(b64, G=[b64.steps // 2] * b64.B)
+    rag = inputs.qwen_ragged(w=w)
+    rag = dataclasses.replace(rag, N=[n + g for n, g in zip(rag.N, rag.G)], G=[0] * rag.B)
+    return {
+        "batch1_30s": (one, f"batch 1, 30 s audio ({one.T[0]} frames), 32-token prompt, "
+                            f"{one.G[0]} of {one.steps} tokens generated"),
+        "batch64_30s": (b64, f"batch 64 x 30 s audio ({b64.T[0]} frames), 32-token prompt, "
+                             f"{b64.G[0]} of {b64.steps} tokens generated"),
+        "ragged128": (rag, "128 requests: audio uniform 5-120 s (63-1500 frames), prompt "
+                           "16-256 tokens, 0-512 tokens generated (one seeded draw)"),
+    }
+
+
+def measure_configs(args, dist: Dist, clocks, peak: float):
+    """Each workload at w = 4 and its uncompressed twin (w = 1, identical
+    seeded tensors), through the same decode step as the headline."""
+    res = {}
+    w4, w1 = config_workloads(4), config_workloads(1)
+    for name in w4:
+        wl, desc = w4[name]
+        r = measure(wl, args.sweep_steps, args.warmup, args.graph_chunk, dist, clocks,
+                    seed_key=0)
+        r1 = measure(w1[name][0], args.sweep_steps, args.warmup, args.graph_chunk, dist, clocks,
+                     seed_key=0)
+        row = {
+            "workload": desc, "B": wl.B, "w": wl.w, "l0": wl.l0,
+            "us_per_step_per_layer": round(r["us_per_step_per_layer"], 3),
+            "step_us": round(r["step_us"], 2),
+            "attn_us_compressed_layer": round(r["attn_us_compressed_layer"], 3),
+            "attn_us_full_layer": round(r["attn_us_full_layer"], 3),
+            "isolated_us_compressed_layer": round(r["isolated_us_compressed_layer"], 2),
+            "w1_us_per_step_per_layer": round(r1["us_per_step_per_layer"], 3),
+            "w1_step_us": round(r1["step_us"], 2),
+            "w1_attn_us_same_layer": round(r1["attn_us_compressed_layer"], 3),
+            "speedup_vs_w1_compressed_layer": round(r1["attn_us_compressed_layer"] /
+                                                    r["attn_us_compressed_layer"], 3),
+            "speedup_vs_w1_step": round(r1["step_us"] / r["step_us"], 3),
+            "steps": args.sweep_steps,
+        }
+        if name == "batch1_30s":
+            row["note"] = ("latency case: each layer's cache is under 1 MB and the whole "
+                           "step's caches stay in L2, so no HBM roofline applies")
+        else:
+            row.update({
+                "attn_gbs_compressed_layer": round(r["attn_gbs_compressed_layer"], 1),
+                "attn_bytes_per_launch_compressed": round(r["attn_bytes_per_launch_compressed"]),
+                "frac_compressed_layer": round(r["attn_gbs_compressed_layer"] / peak, 4),
+                "attn_gbs_full_layer": round(r["attn_gbs_full_layer"], 1),
+                "frac_full_layer": round(r["attn_gbs_full_layer"] / peak, 4),
+                "step_gbs": round(r["step_gbs"], 1),
+                "frac_step": round(r["step_gbs"] / peak, 4),
+            })
+        res[name] = row
+    return res
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and --impl reference): whole decode steps
+# ---------------------------------------------------------------------------
+# A step of the oracle is the same work as a GPU step: for each of the 28
+# layers, every (request, KV head) pair of the batch appends its new token
+# and runs decode attention over its cache (layers < l0 full resolution,
+# the others pooled).  The pairs are split over one worker process per host
+# core (a pool started by spawn); each worker builds its own pairs' caches
+# with the oracle itself (pooling the prefill keys/values) before any timing.
+# Layers of one kind share one cache per pair in the baseline: their
+# arithmetic and row counts are identical, and every layer call writes its
+# token at the step's row and attends over the rows up to it.
+
+_OW = None  # worker state: {"pairs": [...], "L": layers, "l0": l0}
+
+
+def _oracle_worker_init(minutes: int, w: int, seed: int, pairs, steps_total: int):
     import numpy as np
     import oracle
     from paper_2607_06827_gb300 import inputs
+    global _OW
     wl = inputs.qwen_long_audio(minutes, w, generated=GENERATED, seed=seed)
     G = wl.H_q // wl.H_kv
-    out = {}
-    for kind, layer in (("pooled", wl.l0), ("full", 0)):
-        S = wl.P[0] + wl.T[0] + wl.N[0]
-        K = inputs.normal_f32(wl.seed, (90, layer, 0), (S, 1, wl.d)).astype(np.float64)
-        V = inputs.normal_f32(wl.seed, (91, layer, 0), (S, 1, wl.d)).astype(np.float64)
-        u = inputs.normal_f32(wl.seed, (92, layer), (1, wl.d), std=1 / math.sqrt(wl.d))
-        Kc, Vc = oracle.pool_request(K, V, wl.P[0], wl.T[0], wl.N[0], u, wl.w, layer, wl.l0,
-                                     storage=oracle.STORE_BF16)
-        gk = inputs.normal_f32(wl.seed, (93, layer), (wl.G[0] + 1, 1, wl.d)).astype(np.float64)
-        gv = inputs.normal_f32(wl.seed, (94, layer), (wl.G[0] + 1, 1, wl.d)).astype(np.float64)
-        Kc = np.concatenate([Kc, gk]); Vc = np.concatenate([Vc, gv])
-        q = inputs.normal_f32(wl.seed, (95, layer), (G, wl.d)).astype(np.float64)
-        out[kind] = (q, Kc, Vc)
-    return wl, out
+    state = []
+    for b, h in pairs:
+        S = wl.P[b] + wl.T[b] + wl.N[b]
+        per_kind = {}
+        for kind, layer in (("pooled", wl.l0), ("full", 0)):
+            key = (layer, b, h)
+            K = inputs.normal_f32(wl.seed, (90, *key), (S, 1, wl.d)).astype(np.float64)
+            V = inputs.normal_f32(wl.seed, (91, *key), (S, 1, wl.d)).astype(np.float64)
+            u = inputs.normal_f32(wl.seed, (92, *key), (1, wl.d), std=1 / math.sqrt(wl.d))
+            Kp, Vp = oracle.pool_request(K, V, wl.P[b], wl.T[b], wl.N[b], u, wl.w, layer, wl.l0,
+                                         storage=oracle.STORE_BF16)
+            n = Kp.shape[0]
+            cap = n + wl.G[b] + steps_total
+            Kc = np.zeros((cap, 1, wl.d)); Vc = np.zeros_like(Kc)
+            Kc[:n], Vc[:n] = Kp, Vp
+            gk = inputs.normal_f32(wl.seed, (93, *key), (wl.G[b], 1, wl.d)).astype(np.float64)
+            gv = inputs.normal_f32(wl.seed, (94, *key), (wl.G[b], 1, wl.d)).astype(np.float64)
+            Kc[n:n + wl.G[b]], Vc[n:n + wl.G[b]] = gk, gv
+            n += wl.G[b]
+            q = inputs.normal_f32(wl.seed, (95, *key), (steps_total, G, wl.d)).astype(np.float64)
+            kn = inputs.normal_f32(wl.seed, (96, *key), (steps_total, wl.d)).astype(np.float64)
+            vn = inputs.normal_f32(wl.seed, (97, *key), (steps_total, wl.d)).astype(np.float64)
+            per_kind[kind] = (Kc, Vc, n, q, kn.reshape(steps_total, 1, wl.d),
+                              vn.reshape(steps_total, 1, wl.d))
+        state.append(per_kind)
+    _OW = {"pairs": state, "L": wl.L, "l0": wl.l0}
 
 
-def oracle_time_per_step_layer(wl, sample, budget_s: float, max_reps: int | None = None):
-    """Times oracle decode attention on the sample (one KV head of one
-    request) and scales it to the whole batch: us per decode step per layer,
-    averaged over the 28-layer mix (layers < l0 full resolution)."""
+def _oracle_worker_step(step: int, layers) -> float:
+    """One decode step of this worker's pairs over the given layers: append,
+    then attention (oracle, fp64, bf16 storage rounding).  Returns CPU
+    seconds."""
     import oracle
-    t = {}
-    reps = {}
-    for kind in ("pooled", "full"):
-        q, K, V = sample[kind]
-        n, tot = 0, 0.0
-        while True:
-            t0 = time.perf_counter()
-            oracle.decode_attn_request(q, K, V, storage=oracle.STORE_BF16)
-            tot += time.perf_counter() - t0
-            n += 1
-            if tot >= budget_s / 2 or (max_reps and n >= max_reps):
-                break
-        t[kind], reps[kind] = tot / n, n
-    scale = wl.B * wl.H_kv                    # (request, KV head) pairs per layer
-    n_full, n_pooled = wl.l0, wl.L - wl.l0
-    per_layer_s = (t["full"] * n_full + t["pooled"] * n_pooled) / wl.L * scale
-    return per_layer_s * 1e6, t, reps
+    t0 = time.process_time()
+    for layer in layers:
+        kind = "full" if layer < _OW["l0"] else "pooled"
+        for per_kind in _OW["pairs"]:
+            Kc, Vc, n0, q, kn, vn = per_kind[kind]
+            n = oracle.append_request(Kc, Vc, n0 + step, kn[step], vn[step])
+            oracle.decode_attn_request(q[step], Kc[:n], Vc[:n], storage=oracle.STORE_BF16)
+    return time.process_time() - t0
 
 
-_ORACLE_SAMPLE = None
+def _cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return "unknown"
 
 
-def _oracle_worker_init(sample):
-    global _ORACLE_SAMPLE
-    _ORACLE_SAMPLE = sample
+class OracleSteps:
+    """A spawn pool of one worker per host core, each holding its share of
+    the (request, KV head) pairs of the batch; step() runs one whole decode
+    step of the oracle over all of them and returns its wall time."""
+
+    def __init__(self, minutes: int, w: int, steps_total: int, seed: int = 1004):
+        import multiprocessing as mp
+        from paper_2607_06827_gb300 import inputs
+        wl = inputs.qwen_long_audio(minutes, w, generated=GENERATED, seed=seed)
+        self.wl = wl
+        self.cores = os.cpu_count() or 1
+        pairs = [(b, h) for b in range(wl.B) for h in range(wl.H_kv)]
+        self.workers = min(self.cores, len(pairs))
+        shares = [pairs[i::self.workers] for i in range(self.workers)]
+        self.steps_total = steps_total
+        ctx = mp.get_context("spawn")
+        # one single-worker pool per share, so that every share has its own
+        # process (and its own caches)
+        self.pools = [ctx.Pool(1, initializer=_oracle_worker_init,
+                               initargs=(minutes, w, seed, share, steps_total))
+                      for share in shares]
+        for p in self.pools:  # wait until every worker has built its caches
+            p.apply(time.time)
+        self.next = 0
+
+    def step(self, n_layers: int | None = None) -> tuple[float, float, int]:
+        """One decode step over all layers, or over n_layers of them taken in
+        turn (step s starts where step s - 1 stopped, so that bounded runs
+        cover the layer mix in proportion).  Returns (wall s, CPU s, layers)."""
+        if self.next >= self.steps_total:
+            raise RuntimeError("oracle steps exhausted")
+        s = self.next
+        self.next += 1
+        L = self.wl.L
+        n = L if n_layers is None else max(1, min(L, n_layers))
+        layers = [(s * n + j) % L for j in range(n)]
+        t0 = time.perf_counter()
+        res = [p.apply_async(_oracle_worker_step, (s, layers)) for p in self.pools]
+        cpu = sum(r.get() for r in res)
+        return time.perf_counter() - t0, cpu, n
+
+    def close(self):
+        for p in self.pools:
+            p.close()
+            p.join()
+
+    def describe(self, timed_steps: int, layers_per_step: int, warmup: int) -> str:
+        wl = self.wl
+        what = ("whole decode steps" if layers_per_step == wl.L else
+                f"decode steps of {layers_per_step} of the {wl.L} layers each, taken in turn "
+                f"(value = wall time per layer processed)")
+        return (f"{what} of the oracle (plain C, fp64, bf16 storage rounding) on the headline "
+                f"batch: 28 layers ({wl.l0} full resolution, {wl.L - wl.l0} pooled) x "
+                f"{wl.B * wl.H_kv} (request, KV head) pairs, each an append and an attention "
+                f"over its cache; pairs split over {self.workers} worker processes on "
+                f"{self.cores} host cores ({_cpu_model()}); {timed_steps} timed steps after "
+                f"{warmup} untimed; layers of one kind share one cache per pair (same "
+                f"arithmetic and rows)")
 
 
-def _oracle_worker_run(job):
-    """Oracle decode attention, `n` times on the sample's `kind` layer."""
-    import oracle
-    kind, n = job
-    q, K, V = _ORACLE_SAMPLE[kind]
-    for _ in range(n):
-        oracle.decode_attn_request(q, K, V, storage=oracle.STORE_BF16)
-    return n
+def cpu_baseline(timed_steps: int = 3) -> dict:
+    """The oracle as it stands on the host cores: mean wall time of whole
+    decode steps, per step and layer."""
+    o = OracleSteps(HEADLINE_MINUTES, HEADLINE_W, steps_total=timed_steps + 1)
+    try:
+        o.step()
+        walls, cpus, _ = zip(*[o.step() for _ in range(timed_steps)])
+    finally:
+        o.close()
+    wall = sum(walls) / len(walls)
+    return {"value": wall * 1e6 / o.wl.L, "unit": UNIT, "cores": o.workers, "kind": "oracle",
+            "sample": o.describe(timed_steps, o.wl.L, 1), "ms_per_step": round(wall * 1e3, 1),
+            "cpu_seconds": round(sum(cpus), 1)}
 
 
-def cpu_baseline_all_cores(wl, sample, rounds: int = 3):
-    """The same oracle calls over every host core: one layer's (request, KV
-    head) pairs split across a process pool (started by spawn), wall time of
-    the whole layer, best of `rounds`; us per step per layer over the
-    28-layer mix."""
-    import multiprocessing as mp
-    n = os.cpu_count() or 1
-    pairs = wl.B * wl.H_kv
-    chunks = [pairs // n + (1 if i < pairs % n else 0) for i in range(n)]
-    t = {}
-    with mp.get_context("spawn").Pool(n, initializer=_oracle_worker_init,
-                                      initargs=(sample,)) as pool:
-        pool.map(_oracle_worker_run, [("pooled", 1)] * n)  # imports, first touch
-        for kind in ("pooled", "full"):
-            best = math.inf
-            for _ in range(rounds):
-                t0 = time.perf_counter()
-                pool.map(_oracle_worker_run, [(kind, c) for c in chunks if c])
-                best = min(best, time.perf_counter() - t0)
-            t[kind] = best
-    n_full, n_pooled = wl.l0, wl.L - wl.l0
-    us = (t["full"] * n_full + t["pooled"] * n_pooled) / wl.L * 1e6
-    return {"value": us, "unit": UNIT, "cores": n, "kind": "oracle",
-            "sample": (f"oracle decode attention (plain C, fp64) for all {pairs} (request, KV "
-                       f"head) pairs of a pooled and of a full-resolution layer of the headline "
-                       f"workload, split over {n} worker processes; wall time per layer, best of "
-                       f"{rounds}, over the 20 pooled / 8 full layer mix")}
-
-
-def cpu_baseline(budget_s: float):
-    wl, sample = oracle_sample_inputs(HEADLINE_MINUTES, HEADLINE_W)
-    us, t, reps = oracle_time_per_step_layer(wl, sample, budget_s)
-    return {"value": us, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": (f"oracle decode attention (plain C, fp64, single thread) on one KV head "
-                       f"of one request of the headline workload: pooled layer "
-                       f"({sample['pooled'][1].shape[0]} rows) x{reps['pooled']} and "
-                       f"full-resolution layer ({sample['full'][1].shape[0]} rows) "
-                       f"x{reps['full']}; scaled by {wl.B * wl.H_kv} (request, head) pairs "
-                       f"and the 20 pooled / 8 full layer mix"),
-            "all_cores": cpu_baseline_all_cores(wl, sample)}
+# whole oracle steps while W + K stays at or below this; beyond it each step
+# runs a share of the layers so that the reference arm ends within minutes
+REFERENCE_WHOLE_STEPS = 40
 
 
 def run_reference(args):
-    """--impl reference: the CPU oracle, as it stands, on the host cores."""
-    wl, sample = oracle_sample_inputs(args.minutes, args.w)
-    per_step_budget = max(0.05, 150.0 / max(1, args.steps + args.warmup))
-    for _ in range(args.warmup):
-        oracle_time_per_step_layer(wl, sample, per_step_budget, max_reps=1)
-    vals = []
-    t0 = time.time()
-    for _ in range(args.steps):
-        us, _, _ = oracle_time_per_step_layer(wl, sample, per_step_budget, max_reps=1)
-        vals.append(us)
-    wall = time.time() - t0
-    value = sum(vals) / len(vals)
+    """--impl reference: the CPU oracle, as it stands, on the host cores: W
+    untimed and K timed decode steps of the same workload (whole steps up to
+    REFERENCE_WHOLE_STEPS in all, a share of the layers per step beyond)."""
+    total = args.warmup + args.steps
+    o = OracleSteps(args.minutes, args.w, steps_total=total)
+    L = o.wl.L
+    n_layers = L if total <= REFERENCE_WHOLE_STEPS else max(1, L * REFERENCE_WHOLE_STEPS // total)
+    try:
+        for _ in range(args.warmup):
+            o.step(n_layers)
+        runs = [o.step(n_layers) for _ in range(args.steps)]
+    finally:
+        o.close()
+    wall = sum(r[0] for r in runs)
+    layers_done = sum(r[2] for r in runs)
+    value = wall * 1e6 / layers_done                  # us per layer-step, measured
+    ms_per_step = wall * 1e3 / args.steps             # wall time of a timed step
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": value * wl.L / 1e3, "sample_wall_ms_per_step": wall * 1e3 / args.steps,
+        "ms_per_step": ms_per_step, "layers_per_step": n_layers,
         "higher_is_better": False, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(args.minutes, args.w, args.gpus),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": ("each step times oracle decode attention once on one KV "
-                                    "head of one request at a pooled and at a full-resolution "
-                                    "layer, scaled to the batch and the 28-layer mix")},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": o.workers, "kind": "oracle",
+                         "sample": o.describe(args.steps, n_layers, args.warmup)},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(finite_json(line)), flush=True)
@@ -1047,6 +1166,9 @@ def main():
                 "speedup_vs_w1_step": (round(w1["step_us"] / r["step_us"], 3) if w1 else None),
             })
 
+    configs = None
+    if not args.no_configs:
+        configs = measure_configs(args, dist, clocks, measured_peak()[0])
     paged = None
     if not args.no_paged:
         paged = measure_paged(wl, clocks)
@@ -1055,7 +1177,7 @@ def main():
         prefill = measure_prefill(inputs.qwen_long_audio(args.minutes, args.w), clocks)
     cpu = None
     if dist.rank == 0 and dist.world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(args.cpu_seconds)
+        cpu = cpu_baseline(args.cpu_steps)
     clk = clocks.finish() if clocks else None
 
     if dist.rank == 0:
@@ -1095,6 +1217,8 @@ def main():
             },
             "cpu_baseline": cpu,
             "e2e": e2e,
+            "isolated_us_compressed_layer": round(main_res["isolated_us_compressed_layer"], 2),
+            "in_step_us_compressed_layer": round(main_res["attn_us_compressed_layer"], 3),
             "gpu_launches": main_res["gpu_launches"],
             "clocks": clk,
             "breakdown": {k: (round(v, 3) if isinstance(v, float) else v)
@@ -1109,6 +1233,7 @@ def main():
                 "decode_step_28_layers": round(w1_res["step_us"] / main_res["step_us"], 3),
             } if w1_res else None),
             "by_audio_len": sweep or None,
+            "configs": configs,
             "prefill": prefill,
             "paged": paged,
         }
