@@ -206,6 +206,30 @@ __device__ __forceinline__ int atomic_add_acq_rel_gpu(int *p, int v) {
     return old;
 }
 
+// Load with acquire semantics at GPU scope (pairs with release writes of
+// other CTAs: their earlier writes are visible to this thread's later reads).
+__device__ __forceinline__ int ld_acquire_gpu(const int *p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Hint: bring `bytes` (a multiple of 16, 16-byte aligned) of global memory
+// into L2.  No value is read; later reads see whatever the memory holds then.
+__device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+
+// Named CTA barrier `id` over `nthreads` threads (a multiple of 32, whole
+// warps): arrive without waiting, or arrive and wait.  Shared-memory writes
+// made before the arrive are visible to the threads whose sync completes.
+__device__ __forceinline__ void named_bar_arrive(int id, int nthreads) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
 // Orders this thread's earlier generic-proxy shared-memory accesses before
 // later async-proxy (TMA) accesses of the same shared memory.
 __device__ __forceinline__ void fence_proxy_async_shared() {

@@ -118,10 +118,30 @@ __device__ __forceinline__ Piece piece_at(const int64_t *cum, int B, int H_kv, i
     return p;
 }
 
-// CTA (of C) whose unit range [U*c/C, U*(c+1)/C) holds unit u.
-__device__ __forceinline__ int64_t cta_of(int64_t u, int64_t U, int64_t C) {
-    return ((u + 1) * C - 1) / U;
+// The stream-K partition of U units over C CTAs: CTA c owns units
+// [U * c / C, U * (c + 1) / C).
+struct Partition {
+    int64_t U, C;
+    __device__ __forceinline__ int64_t lo(int64_t c) const { return U * c / C; }
+    // the CTA whose range holds unit u (0 <= u < U)
+    __device__ __forceinline__ int64_t cta_of(int64_t u) const { return ((u + 1) * C - 1) / U; }
+};
+// CTAs used for U units on a grid of `grid`: at least kMinUnitsPerCta units
+// each (a small batch spread over every SM would only multiply the partial
+// results each (request, head) has to merge), at most the grid.
+constexpr int64_t kMinUnitsPerCta = 64;
+__device__ __forceinline__ int64_t ctas_for(int64_t U, int64_t grid) {
+    const int64_t n = (U + kMinUnitsPerCta - 1) / kMinUnitsPerCta;
+    return n < grid ? n : grid;
 }
+
+// Tiles a CTA streams into its shared-memory ring before it waits for the
+// previous kernel (programmatic dependent launch with
+// SPEECHKV_OVERLAP_PRIOR).
+#ifndef SPEECHKV_PRE_WAIT_TILES
+#define SPEECHKV_PRE_WAIT_TILES 3
+#endif
+constexpr int kPreWaitTiles = SPEECHKV_PRE_WAIT_TILES;
 
 // kAppend: the decode step fused with the cache update -- each request's new
 // key/value (k_new, v_new) is written as cache row len[b], attended to as that
@@ -174,14 +194,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     if (!overlap) griddep_release();
 
     // ---- 1. per-request lengths (clamped to capacity) and their prefix sums
-    for (int b = tid; b < B; b += blockDim.x) {
-        // with pages, every request has the same capacity (max_blocks blocks)
-        // and these offsets only carry it
-        const int64_t capP = (int64_t)map.max_blocks << map.bs_log2;
-        const int64_t o0 = map.table ? (int64_t)b * capP : cache_off[b];
-        const int64_t o1 = map.table ? (int64_t)(b + 1) * capP : cache_off[b + 1];
+    // Row count, first cache row and capacity of request b, and the row its
+    // new token takes (fused append; -1 if none).
+    auto request_row = [&](int b, int64_t o0, int64_t o1, int64_t L) {
         const int64_t cap = o1 - o0;
-        int64_t L = __ldcg(len + b);  // at L2: another grid's CTA wrote it
         int32_t nr = -1;
         if (cap < 0 || o0 < 0) {
             if (blockIdx.x == 0) report_error(err, SPEECHKV_ERR_INVALID_ARG);
@@ -201,8 +217,27 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         offs[b] = o0;
         if (b == B - 1) offs[B] = o1;
         newrow[b] = nr;
-    }
-    if (tid == 0) {
+    };
+    // with pages, every request has the same capacity (max_blocks blocks) and
+    // the offsets only carry it
+    const int64_t capP = (int64_t)map.max_blocks << map.bs_log2;
+    auto off_of = [&](int b) { return map.table ? (int64_t)b * capP : cache_off[b]; };
+    // inclusive prefix sums of cum[1..B] by one warp (lane `ln`)
+    auto scan_lengths = [&](int ln) {
+        int64_t carry = 0;
+        for (int base = 0; base < B; base += 32) {
+            const int i = base + ln;
+            int64_t v = i < B ? cum[i + 1] : 0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int64_t n = __shfl_up_sync(0xffffffffu, v, o);
+                if (ln >= o) v += n;
+            }
+            if (i < B) cum[i + 1] = carry + v;
+            carry += __shfl_sync(0xffffffffu, v, 31);
+        }
+    };
+    auto init_barriers = [&]() {
         cum[0] = 0;
         flags[0] = 0;  // abort
         for (int s = 0; s < S; s++) {
@@ -214,27 +249,51 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             mbar_init(&free_bar[x], 1);
         }
         fence_mbar_init();
-    }
-    __syncthreads();
-    if (tid < 32) {
-        int64_t carry = 0;
-        for (int base = 0; base < B; base += 32) {
-            const int i = base + tid;
-            int64_t v = i < B ? cum[i + 1] : 0;
+    };
+    constexpr int kFastB = 128;  // batches the producer warp sets up alone
+    if (B <= kFastB) {
+        // The producer warp builds the tables and the barriers by itself and
+        // starts its copies at once; the other warps wait for it on a named
+        // barrier (arrive-only for the producer warp, so it never waits).
+        if (warp == W) {
+            int64_t Lr[kFastB / 32], o0r[kFastB / 32], o1r[kFastB / 32];
 #pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int64_t n = __shfl_up_sync(0xffffffffu, v, o);
-                if (tid >= o) v += n;
+            for (int k = 0; k < kFastB / 32; k++) {  // every load in flight at once
+                const int b = lane + 32 * k;
+                if (b < B) {
+                    Lr[k] = __ldcg(len + b);  // at L2: another grid's CTA wrote it
+                    o0r[k] = off_of(b);
+                    o1r[k] = off_of(b + 1);
+                }
             }
-            if (i < B) cum[i + 1] = carry + v;
-            carry += __shfl_sync(0xffffffffu, v, 31);
+#pragma unroll
+            for (int k = 0; k < kFastB / 32; k++) {
+                const int b = lane + 32 * k;
+                if (b < B) request_row(b, o0r[k], o1r[k], Lr[k]);
+            }
+            __syncwarp();
+            scan_lengths(lane);
+            if (lane == 0) init_barriers();
+            __syncwarp();
+            named_bar_arrive(1, C::kThreads);
+        } else {
+            named_bar_sync(1, C::kThreads);
         }
+    } else {
+        for (int b = tid; b < B; b += blockDim.x)
+            request_row(b, off_of(b), off_of(b + 1), __ldcg(len + b));
+        if (tid == 0) init_barriers();
+        __syncthreads();
+        if (tid < 32) scan_lengths(tid);
+        __syncthreads();
     }
-    __syncthreads();
 
     // ---- 2. this CTA's share of the flat (request, head, row) range
     const int64_t U = (int64_t)H_kv * cum[B];
-    const int64_t Cn = U < (int64_t)gridDim.x ? U : (int64_t)gridDim.x;
+    const int64_t Cn = ctas_for(U, gridDim.x);
+    Partition part;
+    part.U = U;
+    part.C = Cn;
     const int64_t c = blockIdx.x;
     // Work that reads what the previous kernel may produce (k_new, v_new) or
     // writes global memory waits for it.  The producer waits after its first
@@ -300,7 +359,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             griddep_release();
         return;
     }
-    const int64_t u0 = U * c / Cn, u1 = U * (c + 1) / Cn;
+    const int64_t u0 = part.lo(c), u1 = part.lo(c + 1);
 
     if (warp == W) {
         // ================= producer: one lane issues bulk copies ============
@@ -325,10 +384,14 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         int ndeferred = 0;
         bool waited = !overlap;
         auto copy_prior = [&](void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
-            if (waited)
+            if (waited) {
                 bulk_g2s(dst, src, bytes, bar);
-            else
+            } else {
+                // warm L2 meanwhile: a prefetch reads no value, so whatever the
+                // previous kernel writes there is what the copy will see
+                prefetch_l2(src, bytes);
                 deferred[ndeferred++] = Deferred{dst, src, bytes, bar};
+            }
         };
         auto flush_deferred = [&]() {
             griddep_release();
@@ -372,8 +435,9 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             // with kAppend, row nr of this (request, head) comes from k_new/v_new
             const int64_t nr = kAppend ? (int64_t)newrow[p.b] : -1;
             for (int64_t t = p.t0; t < p.t1; t += TR) {
-                // a stage is about to be reused: its queries may be queued
-                if (!waited && issued == S) flush_deferred();
+                // Copies issued before the wait for the previous kernel are
+                // limited to kPreWaitTiles tiles (their queries are queued)
+                if (!waited && issued == kPreWaitTiles) flush_deferred();
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
                 if (flags[0] || !mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, err) ||
@@ -430,122 +494,158 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         // that the done-counter round trip is not on the path of a CTA whose
         // only piece ends with the kernel.
         merge_warp_prior_part();
+        // Partials of up to kBatch pieces (every query head) as one round of
+        // the final merge: slot index c0 + j of this (request, head); this
+        // CTA's own piece (index `mine`) is not loaded.
+        auto load_round = [&](int64_t c0, int64_t clast, int64_t mine, int64_t seg,
+                              float (&bm)[kBatch][G], float (&bl)[kBatch][G],
+                              float (&bo)[kBatch][G][kCols]) {
+#pragma unroll
+            for (int j = 0; j < kBatch; j++) {
+                const bool have = c0 + j <= clast && c0 + j != mine;
+                const float *sp = partials + (c0 + j + seg) * slot_floats;
+#pragma unroll
+                for (int g = 0; g < G; g++) {
+                    bm[j][g] = have ? __ldcg(sp + G * D + g) : -INFINITY;
+                    bl[j][g] = have ? __ldcg(sp + G * D + G + g) : 0.f;
+#pragma unroll
+                    for (int i = 0; i < kCols; i++)
+                        bo[j][g][i] = have ? __ldcg(sp + g * D + lane * kCols + i) : 0.f;
+                }
+            }
+        };
         int64_t k = 0;  // piece index within this CTA
         for (int64_t u = u0; u < u1; k++) {
             const Piece p = piece_at(cum, B, H_kv, u, u1);
             const int x = (int)(k & 1);
+            const int64_t seg = (int64_t)p.b * H_kv + p.h;
+            const bool whole = (p.t0 == 0 && p.t1 == p.L);
+            const int64_t A = (int64_t)H_kv * cum[p.b] + (int64_t)p.h * p.L;
+            const int64_t cfirst = whole ? c : part.cta_of(A);
+            const int64_t clast = whole ? c : part.cta_of(A + p.L - 1);
+            const int others = (int)(clast - cfirst);
             const uint32_t use = (uint32_t)((k >> 1) & 1);
             bool ok = !flags[0] && mbar_wait_bounded(&piece_bar[x], use, err);
             ok = __all_sync(0xffffffffu, ok) && !__shfl_sync(0xffffffffu, flags[0], 0);
             const float *mo = mrg + x * C::kMergeFloats;  // [W][G][D]
             const float *mm = mo + W * G * D;              // [W][G]
             const float *ml = mm + W * G;                  // [W][G]
-            const int64_t seg = (int64_t)p.b * H_kv + p.h;
-            const bool whole = (p.t0 == 0 && p.t1 == p.L);
-            float *slot = partials + (c + seg) * slot_floats;  // o [G][D], m [G], l [G]
+            // this CTA's state of the piece: the consumer warps' states merged
+            float M[G], Ls[G], acc[G][kCols];
             if (ok) {
 #pragma unroll
                 for (int g = 0; g < G; g++) {
-                    float M = -INFINITY;
+                    M[g] = -INFINITY;
 #pragma unroll
-                    for (int w = 0; w < W; w++) M = fmaxf(M, mm[w * G + g]);
-                    float Ls = 0.f, acc[kCols];
+                    for (int w = 0; w < W; w++) M[g] = fmaxf(M[g], mm[w * G + g]);
+                    Ls[g] = 0.f;
 #pragma unroll
-                    for (int i = 0; i < kCols; i++) acc[i] = 0.f;
+                    for (int i = 0; i < kCols; i++) acc[g][i] = 0.f;
 #pragma unroll
                     for (int w = 0; w < W; w++) {
-                        const float sc = fast_exp2(mm[w * G + g] - M);  // idle warp: 0
-                        Ls = fmaf(ml[w * G + g], sc, Ls);
+                        const float sc = fast_exp2(mm[w * G + g] - M[g]);  // idle warp: 0
+                        Ls[g] = fmaf(ml[w * G + g], sc, Ls[g]);
                         const float *src = mo + (w * G + g) * D + lane * kCols;
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[i] = fmaf(src[i], sc, acc[i]);
-                    }
-                    if (whole) {
-                        const float inv = 1.f / Ls;
-#pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[i] *= inv;
-                        store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
-                                                lane * kCols,
-                                            acc);
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < kCols; i++) slot[g * D + lane * kCols + i] = acc[i];
-                        if (lane == 0) {
-                            slot[G * D + g] = M;
-                            slot[G * D + G + g] = Ls;
-                        }
+                        for (int i = 0; i < kCols; i++) acc[g][i] = fmaf(src[i], sc, acc[g][i]);
                     }
                 }
             }
             __syncwarp();
             if (lane == 0) mbar_arrive(&free_bar[x]);  // the buffer may be refilled
             if (ok && !whole) {
-                // the last CTA to finish a piece of this (request, head) merges
-                // all of its pieces (publish this CTA's partial first)
-                const int64_t A = (int64_t)H_kv * cum[p.b] + (int64_t)p.h * p.L;
-                const int64_t cfirst = cta_of(A, U, Cn), clast = cta_of(A + p.L - 1, U, Cn);
+                // Split piece: the CTA that finishes last at this (request,
+                // head) merges every piece.  First peek at the ticket: when all
+                // the other CTAs have published already, this one is last and
+                // merges straight from its registers.  Otherwise publish this
+                // partial, then take a ticket (acquire-release) to find out.
                 int last = 0;
-                if (lane == 0)
-                    last = atomic_add_acq_rel_gpu(&counters[seg], 1) == (int)(clast - cfirst);
+                if (lane == 0) last = ld_acquire_gpu(&counters[seg]) == others;
                 last = __shfl_sync(0xffffffffu, last, 0);
-                __syncwarp();  // lane 0's acquire orders the other lanes' reads too
-                if (last) {
-                    // online log-sum-exp over the pieces, per query head g;
-                    // kBatch partials (all heads) in flight per round
-                    float M[G], Ls[G], acc[G][kCols];
+                if (!last) {
+                    float *slot = partials + (c + seg) * slot_floats;  // o [G][D], m [G], l [G]
 #pragma unroll
                     for (int g = 0; g < G; g++) {
-                        M[g] = -INFINITY;
-                        Ls[g] = 0.f;
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[g][i] = 0.f;
+                        for (int i = 0; i < kCols; i++) slot[g * D + lane * kCols + i] = acc[g][i];
+                        if (lane == 0) {
+                            slot[G * D + g] = M[g];
+                            slot[G * D + G + g] = Ls[g];
+                        }
+                    }
+                    __syncwarp();  // the lanes' partial writes precede lane 0's release
+                    if (lane == 0) last = atomic_add_acq_rel_gpu(&counters[seg], 1) == others;
+                    last = __shfl_sync(0xffffffffu, last, 0);
+                }
+                __syncwarp();  // lane 0's acquire orders the other lanes' reads too
+                if (last) {
+                    // online log-sum-exp over the pieces in CTA order (this
+                    // CTA's own state taken from registers in its turn), per
+                    // query head g, so that the result does not depend on which
+                    // CTA came last; kBatch partials (all heads) in flight per
+                    // round
+                    float Mt[G], Lt[G], at[G][kCols];
+#pragma unroll
+                    for (int g = 0; g < G; g++) {
+                        Mt[g] = -INFINITY;
+                        Lt[g] = 0.f;
+#pragma unroll
+                        for (int i = 0; i < kCols; i++) at[g][i] = 0.f;
                     }
 #pragma unroll 1
                     for (int64_t c0 = cfirst; c0 <= clast; c0 += kBatch) {
                         float bm[kBatch][G], bl[kBatch][G], bo[kBatch][G][kCols];
+                        load_round(c0, clast, c, seg, bm, bl, bo);
 #pragma unroll
-                        for (int j = 0; j < kBatch; j++) {
-                            const bool have = c0 + j <= clast;
-                            const float *sp = partials + (c0 + j + seg) * slot_floats;
+                        for (int j = 0; j < kBatch; j++) {  // this CTA's own state
+                            if (c0 + j != c) continue;
 #pragma unroll
                             for (int g = 0; g < G; g++) {
-                                bm[j][g] = have ? __ldcg(sp + G * D + g) : -INFINITY;
-                                bl[j][g] = have ? __ldcg(sp + G * D + G + g) : 0.f;
+                                bm[j][g] = M[g];
+                                bl[j][g] = Ls[g];
 #pragma unroll
-                                for (int i = 0; i < kCols; i++)
-                                    bo[j][g][i] = have ? __ldcg(sp + g * D + lane * kCols + i) : 0.f;
+                                for (int i = 0; i < kCols; i++) bo[j][g][i] = acc[g][i];
                             }
                         }
 #pragma unroll
                         for (int g = 0; g < G; g++) {
-                            float Mn = M[g];
+                            float Mn = Mt[g];
 #pragma unroll
                             for (int j = 0; j < kBatch; j++) Mn = fmaxf(Mn, bm[j][g]);
-                            const float r = fast_exp2(M[g] - Mn);  // 0 while M = -inf
-                            Ls[g] *= r;
+                            const float r = fast_exp2(Mt[g] - Mn);  // 0 while Mt = -inf
+                            Lt[g] *= r;
 #pragma unroll
-                            for (int i = 0; i < kCols; i++) acc[g][i] *= r;
+                            for (int i = 0; i < kCols; i++) at[g][i] *= r;
 #pragma unroll
                             for (int j = 0; j < kBatch; j++) {
                                 const float sc = fast_exp2(bm[j][g] - Mn);  // absent: 0
-                                Ls[g] = fmaf(bl[j][g], sc, Ls[g]);
+                                Lt[g] = fmaf(bl[j][g], sc, Lt[g]);
 #pragma unroll
                                 for (int i = 0; i < kCols; i++)
-                                    acc[g][i] = fmaf(bo[j][g][i], sc, acc[g][i]);
+                                    at[g][i] = fmaf(bo[j][g][i], sc, at[g][i]);
                             }
-                            M[g] = Mn;
+                            Mt[g] = Mn;
                         }
                     }
 #pragma unroll
                     for (int g = 0; g < G; g++) {
-                        const float inv = 1.f / Ls[g];
+                        Ls[g] = Lt[g];
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) acc[g][i] *= inv;
-                        store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
-                                                lane * kCols,
-                                            acc[g]);
+                        for (int i = 0; i < kCols; i++) acc[g][i] = at[g][i];
                     }
-                    if (lane == 0) counters[seg] = 0;
+                    if (lane == 0) counters[seg] = 0;  // ready for the next call
+                }
+                ok = last;
+            }
+            if (ok) {  // a whole piece, or the last CTA of a split one
+#pragma unroll
+                for (int g = 0; g < G; g++) {
+                    const float inv = 1.f / Ls[g];
+#pragma unroll
+                    for (int i = 0; i < kCols; i++) acc[g][i] *= inv;
+                    store_vec<T, kCols>(out + ((int64_t)p.b * H_q + p.h * G + g) * D +
+                                            lane * kCols,
+                                        acc[g]);
                 }
             }
             u += p.t1 - p.t0;
@@ -615,16 +715,22 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                     }
             }
             const unsigned char *vs = ks + C::kTileBytes;
-            const int r0 = warp * RW;
-            int nw = rows - r0;
-            nw = nw < 0 ? 0 : (nw > RW ? RW : nw);
+            // the warp's rows of the tile are interleaved (tile row warp + W j
+            // for its row j), so that a partial tile is shared by every warp
+            // and costs in proportion to its rows
+            const int nw = rows > warp ? (rows - warp + W - 1) / W : 0;
             if (nw > 0 && !aborted) {
                 // ---- scores (q * log2e/sqrt(d)) . k, two packed partial sums
                 float s[G][C::kQkPasses];
 #pragma unroll
                 for (int rr = 0; rr < C::kQkPasses; rr++) {
                     const int row = rr * 8 + lrow;
-                    const unsigned char *kr = ks + (r0 + row) * C::kRowBytes;
+                    if (rr * 8 >= nw) {  // no row of this pass (warp-uniform)
+#pragma unroll
+                        for (int g = 0; g < G; g++) s[g][rr] = -INFINITY;
+                        continue;
+                    }
+                    const unsigned char *kr = ks + (warp + W * row) * C::kRowBytes;
                     float2 acc[G];
 #pragma unroll
                     for (int g = 0; g < G; g++) acc[g] = make_float2(0.f, 0.f);
@@ -674,13 +780,13 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 }
                 __syncwarp();
                 // ---- o += p * v over the warp's valid rows
-                const unsigned char *vw = vs + r0 * C::kRowBytes + pc * 16;
+                const unsigned char *vw = vs + warp * C::kRowBytes + pc * 16;
 #pragma unroll 4
                 for (int j0 = 0; j0 < nw; j0 += C::kPvRowsPerPass) {
                     const int row = j0 + pr;
                     if (row < nw) {
                         float2 v2[C::kPairsPerChunk];
-                        load16_pairs<T>(vw + row * C::kRowBytes, v2);
+                        load16_pairs<T>(vw + row * (W * C::kRowBytes), v2);
 #pragma unroll
                         for (int g = 0; g < G; g++) {
                             const float2 pg = pw[row * G + g];
