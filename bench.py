@@ -615,8 +615,17 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
     return res
 
 
-def measure_paged(wl, clocks, block_size: int = 64, steps: int = 64, warmup: int = 4,
-                  chunk: int = 32):
+PAGE_SIZES = (16, 32, 64)  # rows per page of the paged-cache measurement
+
+
+def measure_paged(wl, clocks, steps: int = 64, warmup: int = 4, chunk: int = 32):
+    """speechkv_decode_step_paged against speechkv_decode_step for pages of
+    16, 32 and 64 rows (16 is vLLM's default)."""
+    return {"steps": steps, "by_block_size": [
+        measure_paged_one(wl, clocks, bs, steps, warmup, chunk) for bs in PAGE_SIZES]}
+
+
+def measure_paged_one(wl, clocks, block_size: int, steps: int, warmup: int, chunk: int):
     """speechkv_decode_step_paged against speechkv_decode_step on the same
     layer (one pooled, one full-resolution), same inputs: pages of
     block_size rows in a shuffled block table.  Each path runs `steps` fused
@@ -624,7 +633,7 @@ def measure_paged(wl, clocks, block_size: int = 64, steps: int = 64, warmup: int
     import numpy as np
     import torch
     from paper_2607_06827_gb300 import inputs, speechkv as sk
-    res = {"block_size": block_size, "steps": steps}
+    res = {"block_size": block_size}
     B, Hq, Hk, d = wl.B, wl.H_q, wl.H_kv, wl.d
     full_rows = wl.full_rows()
     full_off = torch.from_numpy(np.concatenate([[0], np.cumsum(full_rows)]).astype(np.int64)).cuda()

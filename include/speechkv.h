@@ -382,8 +382,9 @@ speechkv_status speechkv_decode_step_noalloc(
  * block_size   a power of two; each request's capacity is
  *              max_blocks * block_size rows (at most 2^31 - 1).  The
  *              decode step reads a 128-row tile as one copy per page
- *              segment: pages of 64 rows or more keep it within ~7 % of
- *              the contiguous layout; 16-row pages cost up to ~1.8x.
+ *              segment, the segments issued in parallel: measured against
+ *              the contiguous layout, 64-row pages cost 2-4 %, 16-row pages
+ *              (vLLM's default) 4-12 %.
  * num_blocks   host: pages in k_pages / v_pages (bounds the table entries).
  * The other arguments, the results and the errors are those of the
  * contiguous entry point of the same name (the rows and their order are the

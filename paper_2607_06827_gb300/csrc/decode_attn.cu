@@ -362,16 +362,17 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     const int64_t u0 = part.lo(c), u1 = part.lo(c + 1);
 
     if (warp == W) {
-        // ================= producer: one lane issues bulk copies ============
-        // lanes 1..31 leave at once: a grid dependency wait on this warp would
-        // also hold lane 0 back (the other warps' waits order the CTA's exit)
-        if (lane != 0) return;
+        // ================= producer warp =====================================
+        // Lane 0 drives the ring (waits, expected bytes, queries, new rows);
+        // with a block table, every lane copies its own page segments of a
+        // tile, so small pages cost no more issue time than large ones.  The
+        // control flow is warp-uniform (lane 0's decisions are broadcast).
         int stage = 0;
         uint32_t phase = 0;
         int64_t issued = 0;
         bool stop = false;
         // Copies of data the previous kernel may produce (queries, new
-        // tokens) wait for it; until then they are queued here.  Only the
+        // tokens) wait for it; until then lane 0 queues them here.  Only the
         // first S tiles can be issued before the first stage must be reused,
         // so the queue holds at most 3 copies per stage.
         struct Deferred {
@@ -384,6 +385,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         int ndeferred = 0;
         bool waited = !overlap;
         auto copy_prior = [&](void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+            if (lane != 0) return;
             if (waited) {
                 bulk_g2s(dst, src, bytes, bar);
             } else {
@@ -396,8 +398,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         auto flush_deferred = [&]() {
             griddep_release();
             waited = true;
-            for (int i = 0; i < ndeferred; i++)
-                bulk_g2s(deferred[i].dst, deferred[i].src, deferred[i].bytes, deferred[i].bar);
+            if (lane == 0)
+                for (int i = 0; i < ndeferred; i++)
+                    bulk_g2s(deferred[i].dst, deferred[i].src, deferred[i].bytes,
+                             deferred[i].bar);
             ndeferred = 0;
         };
         for (int64_t u = u0; u < u1 && !stop;) {
@@ -406,30 +410,32 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             const int64_t base = offs[p.b] * H_kv + (int64_t)p.h * cap;
             // Rows [t_from, t_from + nrows) of this (request, head) into the
             // stage (keys at dst, values kTileBytes further): one bulk copy per
-            // tensor for a contiguous run, one per page segment with a block
-            // table.  An invalid page is reported and read from page 0 instead
-            // (the stage's byte count must still arrive).
+            // tensor for a contiguous run (lane 0), one per page segment with a
+            // block table (lane i takes segments i, i + 32, ...).  An invalid
+            // page is reported and read from page 0 instead (the stage's byte
+            // count must still arrive).
             auto copy_rows = [&](unsigned char *dst, int64_t t_from, int64_t nrows, uint64_t *bar) {
                 if (!map.table) {
+                    if (lane != 0) return;
                     const uint32_t bytes = (uint32_t)nrows * C::kRowBytes;
                     bulk_g2s(dst, kc + (base + t_from) * D, bytes, bar);
                     bulk_g2s(dst + C::kTileBytes, vc + (base + t_from) * D, bytes, bar);
                     return;
                 }
-                const int64_t bs = 1ll << map.bs_log2;
-                for (int64_t tt = t_from; tt < t_from + nrows;) {
-                    const int64_t left = t_from + nrows - tt, room = bs - (tt & (bs - 1));
-                    const int64_t seg = left < room ? left : room;
-                    int64_t off = cache_row(map, p.b, p.h, tt, H_kv, D, 0, 0);
+                const int lg = map.bs_log2;
+                const int64_t t_end = t_from + nrows;
+                for (int64_t pg = (t_from >> lg) + lane; pg <= (t_end - 1) >> lg; pg += 32) {
+                    const int64_t s0 = (pg << lg) > t_from ? (pg << lg) : t_from;
+                    const int64_t s1 = ((pg + 1) << lg) < t_end ? ((pg + 1) << lg) : t_end;
+                    int64_t off = cache_row(map, p.b, p.h, s0, H_kv, D, 0, 0);
                     if (off < 0) {
                         report_error(err, SPEECHKV_ERR_INVALID_ARG);
                         off = 0;
                     }
-                    const uint32_t at = (uint32_t)(tt - t_from) * C::kRowBytes;
-                    const uint32_t bytes = (uint32_t)seg * C::kRowBytes;
+                    const uint32_t at = (uint32_t)(s0 - t_from) * C::kRowBytes;
+                    const uint32_t bytes = (uint32_t)(s1 - s0) * C::kRowBytes;
                     bulk_g2s(dst + at, kc + off, bytes, bar);
                     bulk_g2s(dst + C::kTileBytes + at, vc + off, bytes, bar);
-                    tt += seg;
                 }
             };
             // with kAppend, row nr of this (request, head) comes from k_new/v_new
@@ -440,9 +446,13 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 if (!waited && issued == kPreWaitTiles) flush_deferred();
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
-                if (flags[0] || !mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, err) ||
-                    flags[0]) {
-                    flags[0] = 1;
+                int ok = 1;
+                if (lane == 0)
+                    ok = !flags[0] && mbar_wait_bounded(&empty_bar[stage], phase ^ 1u, err) &&
+                         !flags[0];
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) {
+                    if (lane == 0) flags[0] = 1;
                     stop = true;
                     break;
                 }
@@ -450,7 +460,9 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                 const uint32_t bytes = (uint32_t)rows * C::kRowBytes;
                 const bool first = (t == p.t0);
                 unsigned char *dst = stages + (size_t)stage * C::kStageBytes;
-                mbar_arrive_expect_tx(&full_bar[stage], 2 * bytes + (first ? C::kQBytes : 0));
+                if (lane == 0)
+                    mbar_arrive_expect_tx(&full_bar[stage], 2 * bytes + (first ? C::kQBytes : 0));
+                __syncwarp();
                 if (kAppend && nr >= t && nr < t + rows) {
                     // the tile ends with the new token: cached rows, then one
                     // row from k_new / v_new (always the last row of the run)
@@ -476,9 +488,11 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         }
         if (!waited) flush_deferred();
         // Let the copies still in flight land before the CTA may exit.
-        const int64_t first = issued > S ? issued - S : 0;
-        for (int64_t k = first; k < issued; k++)
-            if (!mbar_wait_bounded(&full_bar[k % S], (uint32_t)((k / S) & 1), err)) break;
+        if (lane == 0) {
+            const int64_t first = issued > S ? issued - S : 0;
+            for (int64_t k = first; k < issued; k++)
+                if (!mbar_wait_bounded(&full_bar[k % S], (uint32_t)((k / S) & 1), err)) break;
+        }
         return;
     }
 
