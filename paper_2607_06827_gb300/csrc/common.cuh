@@ -220,16 +220,6 @@ __device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
-// Named CTA barrier `id` over `nthreads` threads (a multiple of 32, whole
-// warps): arrive without waiting, or arrive and wait.  Shared-memory writes
-// made before the arrive are visible to the threads whose sync completes.
-__device__ __forceinline__ void named_bar_arrive(int id, int nthreads) {
-    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
-__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
-    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
-}
-
 // Orders this thread's earlier generic-proxy shared-memory accesses before
 // later async-proxy (TMA) accesses of the same shared memory.
 __device__ __forceinline__ void fence_proxy_async_shared() {

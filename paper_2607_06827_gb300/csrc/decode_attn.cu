@@ -146,7 +146,9 @@ constexpr int kPreWaitTiles = SPEECHKV_PRE_WAIT_TILES;
 // kAppend: the decode step fused with the cache update -- each request's new
 // key/value (k_new, v_new) is written as cache row len[b], attended to as that
 // row (copied straight from k_new/v_new), and len[b] advances by one.
-template <typename T, int D, int G, bool kAppend>
+// kPaged: the cache is paged through map's block table (its own instance, so
+// that the contiguous kernel carries none of that code).
+template <typename T, int D, int G, bool kAppend, bool kPaged>
 __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, G>::kCtasPerSm)
     decode_attn_kernel(const T *__restrict__ q, const T *__restrict__ k_new,
                        const T *__restrict__ v_new, T *__restrict__ kc, T *__restrict__ vc,
@@ -221,7 +223,7 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     // with pages, every request has the same capacity (max_blocks blocks) and
     // the offsets only carry it
     const int64_t capP = (int64_t)map.max_blocks << map.bs_log2;
-    auto off_of = [&](int b) { return map.table ? (int64_t)b * capP : cache_off[b]; };
+    auto off_of = [&](int b) { return kPaged ? (int64_t)b * capP : cache_off[b]; };
     // inclusive prefix sums of cum[1..B] by one warp (lane `ln`)
     auto scan_lengths = [&](int ln) {
         int64_t carry = 0;
@@ -250,43 +252,12 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         }
         fence_mbar_init();
     };
-    constexpr int kFastB = 128;  // batches the producer warp sets up alone
-    if (B <= kFastB) {
-        // The producer warp builds the tables and the barriers by itself and
-        // starts its copies at once; the other warps wait for it on a named
-        // barrier (arrive-only for the producer warp, so it never waits).
-        if (warp == W) {
-            int64_t Lr[kFastB / 32], o0r[kFastB / 32], o1r[kFastB / 32];
-#pragma unroll
-            for (int k = 0; k < kFastB / 32; k++) {  // every load in flight at once
-                const int b = lane + 32 * k;
-                if (b < B) {
-                    Lr[k] = __ldcg(len + b);  // at L2: another grid's CTA wrote it
-                    o0r[k] = off_of(b);
-                    o1r[k] = off_of(b + 1);
-                }
-            }
-#pragma unroll
-            for (int k = 0; k < kFastB / 32; k++) {
-                const int b = lane + 32 * k;
-                if (b < B) request_row(b, o0r[k], o1r[k], Lr[k]);
-            }
-            __syncwarp();
-            scan_lengths(lane);
-            if (lane == 0) init_barriers();
-            __syncwarp();
-            named_bar_arrive(1, C::kThreads);
-        } else {
-            named_bar_sync(1, C::kThreads);
-        }
-    } else {
-        for (int b = tid; b < B; b += blockDim.x)
-            request_row(b, off_of(b), off_of(b + 1), __ldcg(len + b));
-        if (tid == 0) init_barriers();
-        __syncthreads();
-        if (tid < 32) scan_lengths(tid);
-        __syncthreads();
-    }
+    for (int b = tid; b < B; b += blockDim.x)
+        request_row(b, off_of(b), off_of(b + 1), __ldcg(len + b));  // len at L2: another grid wrote it
+    if (tid == 0) init_barriers();
+    __syncthreads();
+    if (tid < 32) scan_lengths(tid);
+    __syncthreads();
 
     // ---- 2. this CTA's share of the flat (request, head, row) range
     const int64_t U = (int64_t)H_kv * cum[B];
@@ -340,7 +311,9 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
                     const int e = (i - tensor * nvec) * kVec;
                     const int hh = e / D, col = e - hh * D;
                     const T *src = (tensor ? v_new : k_new) + (int64_t)b * H_kv * D + e;
-                    const int64_t row = cache_row(map, b, hh, nr, H_kv, D, offs[b], cap);
+                    const int64_t row =
+                        kPaged ? cache_row(map, b, hh, nr, H_kv, D, 0, 0)
+                               : (offs[b] * H_kv + (int64_t)hh * cap + nr) * D;
                     if (row < 0) {  // invalid page: reported, not written
                         report_error(err, SPEECHKV_ERR_INVALID_ARG);
                         continue;
@@ -415,27 +388,27 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             // page is reported and read from page 0 instead (the stage's byte
             // count must still arrive).
             auto copy_rows = [&](unsigned char *dst, int64_t t_from, int64_t nrows, uint64_t *bar) {
-                if (!map.table) {
+                if constexpr (!kPaged) {
                     if (lane != 0) return;
                     const uint32_t bytes = (uint32_t)nrows * C::kRowBytes;
                     bulk_g2s(dst, kc + (base + t_from) * D, bytes, bar);
                     bulk_g2s(dst + C::kTileBytes, vc + (base + t_from) * D, bytes, bar);
-                    return;
-                }
-                const int lg = map.bs_log2;
-                const int64_t t_end = t_from + nrows;
-                for (int64_t pg = (t_from >> lg) + lane; pg <= (t_end - 1) >> lg; pg += 32) {
-                    const int64_t s0 = (pg << lg) > t_from ? (pg << lg) : t_from;
-                    const int64_t s1 = ((pg + 1) << lg) < t_end ? ((pg + 1) << lg) : t_end;
-                    int64_t off = cache_row(map, p.b, p.h, s0, H_kv, D, 0, 0);
-                    if (off < 0) {
-                        report_error(err, SPEECHKV_ERR_INVALID_ARG);
-                        off = 0;
+                } else {
+                    const int lg = map.bs_log2;
+                    const int64_t t_end = t_from + nrows;
+                    for (int64_t pg = (t_from >> lg) + lane; pg <= (t_end - 1) >> lg; pg += 32) {
+                        const int64_t s0 = (pg << lg) > t_from ? (pg << lg) : t_from;
+                        const int64_t s1 = ((pg + 1) << lg) < t_end ? ((pg + 1) << lg) : t_end;
+                        int64_t off = cache_row(map, p.b, p.h, s0, H_kv, D, 0, 0);
+                        if (off < 0) {
+                            report_error(err, SPEECHKV_ERR_INVALID_ARG);
+                            off = 0;
+                        }
+                        const uint32_t at = (uint32_t)(s0 - t_from) * C::kRowBytes;
+                        const uint32_t bytes = (uint32_t)(s1 - s0) * C::kRowBytes;
+                        bulk_g2s(dst + at, kc + off, bytes, bar);
+                        bulk_g2s(dst + C::kTileBytes + at, vc + off, bytes, bar);
                     }
-                    const uint32_t at = (uint32_t)(s0 - t_from) * C::kRowBytes;
-                    const uint32_t bytes = (uint32_t)(s1 - s0) * C::kRowBytes;
-                    bulk_g2s(dst + at, kc + off, bytes, bar);
-                    bulk_g2s(dst + C::kTileBytes + at, vc + off, bytes, bar);
                 }
             };
             // with kAppend, row nr of this (request, head) comes from k_new/v_new
@@ -865,10 +838,10 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
     griddep_release();
 }
 
-template <typename T, int D, int G, bool kAppend>
+template <typename T, int D, int G, bool kAppend, bool kPaged>
 cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) {
     using C = DecodeCfg<T, D, G>;
-    auto kern = decode_attn_kernel<T, D, G, kAppend>;
+    auto kern = decode_attn_kernel<T, D, G, kAppend, kPaged>;
     static int configured_device_mask = 0;  // devices with the smem attributes set
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -910,7 +883,7 @@ cudaError_t launch_instance(const DecodeArgs &a, int grid, cudaStream_t stream) 
 template <typename T, int D, int G>
 int occupancy_instance(int B) {
     using C = DecodeCfg<T, D, G>;
-    auto kern = decode_attn_kernel<T, D, G, false>;
+    auto kern = decode_attn_kernel<T, D, G, false, false>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)C::smem_bytes(SPEECHKV_MAX_BATCH)) != cudaSuccess ||
         cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100) !=
@@ -957,10 +930,13 @@ int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B) {
 cudaError_t launch_decode(const DecodeArgs &a, int grid, cudaStream_t stream) {
     const int group = a.H_q / a.H_kv;
     const bool append = a.k_new != nullptr;
-#define X(T, D, G)                                                               \
-    if (a.dtype == dtype_of<T>() && a.d == D && group == G)                      \
-        return append ? launch_instance<T, D, G, true>(a, grid, stream)          \
-                      : launch_instance<T, D, G, false>(a, grid, stream);
+    // the paged layout comes with the fused append only (speechkv_decode_step_paged)
+    if (a.map.table && !append) return cudaErrorInvalidValue;
+#define X(T, D, G)                                                                   \
+    if (a.dtype == dtype_of<T>() && a.d == D && group == G)                          \
+        return !append ? launch_instance<T, D, G, false, false>(a, grid, stream)     \
+               : a.map.table ? launch_instance<T, D, G, true, true>(a, grid, stream) \
+                             : launch_instance<T, D, G, true, false>(a, grid, stream);
     SPEECHKV_DECODE_CASES(X)
 #undef X
     return cudaErrorInvalidValue;
