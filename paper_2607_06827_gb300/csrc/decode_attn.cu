@@ -345,16 +345,18 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
         int64_t issued = 0;
         bool stop = false;
         // Copies of data the previous kernel may produce (queries, new
-        // tokens) wait for it; until then lane 0 queues them here.  Only the
-        // first S tiles can be issued before the first stage must be reused,
-        // so the queue holds at most 3 copies per stage.
+        // tokens) wait for it; until then lane 0 queues them here, at most 3
+        // per tile.  No more tiles than the ring holds are issued before the
+        // wait: the next one would wait for a stage whose queries are queued
+        // behind it.
+        constexpr int kPre = kPreWaitTiles < S ? kPreWaitTiles : S;
         struct Deferred {
             void *dst;
             const void *src;
             uint32_t bytes;
             uint64_t *bar;
         };
-        Deferred deferred[3 * S];
+        Deferred deferred[3 * kPre];
         int ndeferred = 0;
         bool waited = !overlap;
         auto copy_prior = [&](void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
@@ -415,8 +417,8 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             const int64_t nr = kAppend ? (int64_t)newrow[p.b] : -1;
             for (int64_t t = p.t0; t < p.t1; t += TR) {
                 // Copies issued before the wait for the previous kernel are
-                // limited to kPreWaitTiles tiles (their queries are queued)
-                if (!waited && issued == kPreWaitTiles) flush_deferred();
+                // limited to kPre tiles (their queries are queued)
+                if (!waited && issued == kPre) flush_deferred();
                 // (re-check the abort flag after the wait: aborted consumers
                 // release stages without waiting for their copies)
                 int ok = 1;

@@ -517,15 +517,16 @@ def test_max_batch_fused_step(sk, oracle):
         H.assert_close(H.f64(out[b]), ref, "bf16", f"request {b}")
 
 
-@pytest.mark.parametrize("grid", [0, 7, 16])
-def test_overlap_prior_two_layer_interleave_any_grid(sk, oracle, grid):
+@pytest.mark.parametrize("grid,H_kv", [(0, 8), (7, 8), (16, 8), (0, 4), (7, 4), (7, 16)])
+def test_overlap_prior_two_layer_interleave_any_grid(sk, oracle, grid, H_kv):
     """SPEECHKV_OVERLAP_PRIOR with the steps of two layers interleaved
     [a, b, a, b, ...]: the kernel two launches back writes this call's cache
     and length.  A decode kernel releases its successor only after its own
     wait for its predecessor, so that kernel has completed before this one
     starts, whatever the grid -- small explicit grids, under which several
     grids fit on the GPU at once, included."""
-    wl = inputs.qwen_ragged(B=5)
+    # H_kv 4 / 16 with 16 query heads: groups of 4 (a two-stage ring) and 1
+    wl = dataclasses.replace(inputs.qwen_ragged(B=5), H_kv=H_kv)
     layers, steps = [wl.l0 - 1, wl.l0], 4
     gl, ol = [], []
     for layer in layers:
@@ -613,3 +614,19 @@ def test_batch64_30s_pool_and_fused_steps(sk, oracle, w):
     pooling -> appends -> attention."""
     wl = inputs.qwen_batch64(w=w)
     _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=3, fused=True)
+
+
+@pytest.mark.parametrize("H_kv,grid", [(8, 0), (8, 1), (8, 3), (4, 0), (4, 5), (16, 0), (16, 2)])
+def test_short_requests_share_tiles(sk, oracle, H_kv, grid):
+    """Many short requests (0-20 rows, some empty) so that a 128-row tile
+    holds the ends and starts of several (request, KV head) runs: tiles are
+    cut before a third run would start in them, and pieces of one row occur.
+    Fused steps against the oracle's pooling -> append -> attention."""
+    rng = np.random.default_rng(77 + H_kv + grid)
+    B = 40
+    T = [int(x) for x in rng.integers(0, 12, B)]
+    N = [int(x) for x in rng.integers(0, 9, B)]
+    T[3] = N[3] = 0                      # an empty request (its rows come from the steps)
+    wl = inputs.Workload(name="short", dtype="bf16", L=1, l0=0, w=4, H_q=16, H_kv=H_kv, d=128,
+                         P=[0] * B, T=T, N=N, G=[0] * B, steps=2, seed=78)
+    _run_steps(sk, oracle, wl, layers=[0], steps=2, fused=True, grid=grid)
