@@ -413,6 +413,9 @@ def measure(wl, steps: int, warmup: int, chunk: int, dist: Dist, clocks, seed_ke
         "attn_bytes_per_launch_compressed": per_kind["compressed"][2],
         "attn_us_full_layer": per_kind["full"][0],
         "attn_gbs_full_layer": per_kind["full"][1],
+        "attn_bytes_per_launch_full": per_kind["full"][2],
+        "n_compressed_layers": len(comp),
+        "n_full_layers": len(full),
         "isolated_us_compressed_layer": isolated["compressed"],
         "isolated_us_full_layer": isolated["full"],
         "isolated_note": (f"one layer's step alone (a one-launch CUDA graph) after reading "
@@ -1046,6 +1049,11 @@ def workload_config(minutes: int, w: int, n_gpus: int) -> dict:
     }
 
 
+def int_or_none(x: float):
+    """round(x), or None when x is not finite (a pass with no layer of a kind)."""
+    return round(x) if math.isfinite(x) else None
+
+
 def finite_json(x):
     """Replace NaN/inf (not valid JSON) by None, recursively."""
     if isinstance(x, float):
@@ -1084,12 +1092,12 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(bytes_per_launch: float):
-    """DRAM bytes per decode-attention launch of this workload, from the
-    committed ncu capture (one pooled layer), scaled by the rows processed:
-    captured traffic x (this workload's algorithmic bytes per launch / the
-    captured launch's algorithmic bytes).  None when the capture was taken on
-    another kernel source."""
+def profiled_traffic(res: dict):
+    """DRAM bytes per decode-attention launch of this workload's step, from the
+    committed ncu captures of one pooled and one full-resolution launch: each
+    kind's traffic / algorithmic-bytes ratio times this workload's
+    algorithmic bytes per launch of that kind, averaged over the step's layer
+    mix.  None when the captures were taken on another kernel source."""
     try:
         kv = {}
         with open(PROFILE_TRAFFIC) as f:
@@ -1099,8 +1107,15 @@ def profiled_traffic(bytes_per_launch: float):
                     kv[k.strip()] = v.strip()
         if kv.get("kernel_sha256_16") != kernel_hash():
             return None
-        scale = bytes_per_launch / float(kv["algorithmic_bytes"])
-        return round(float(kv["dram_bytes_per_launch"]) * scale)
+        total, n = 0.0, 0
+        for kind, key in (("pooled", "compressed"), ("full", "full")):
+            count = res[f"n_{key}_layers"]
+            if not count:
+                continue
+            ratio = float(kv[f"{kind}_dram_bytes_per_launch"]) / float(kv[f"{kind}_algorithmic_bytes"])
+            total += count * ratio * res[f"attn_bytes_per_launch_{key}"]
+            n += count
+        return round(total / n) if n else None
     except (OSError, ValueError, KeyError, ZeroDivisionError):
         return None
 
@@ -1209,7 +1224,7 @@ def main():
             "roofline": {
                 "bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "peak_kind": peak_kind,
-                "traffic": profiled_traffic(main_res["attn_bytes_per_launch_all"]),
+                "traffic": profiled_traffic(main_res),
                 "kernel": ("decode_attn_kernel (fused append, bf16, d=128, group 2) of "
                            "speechkv_decode_step: the only kernel of the step"),
                 "achieved_from": "algorithmic bytes of all launches of the timed steps / "
@@ -1221,7 +1236,7 @@ def main():
                     "frac": round(main_res["attn_gbs_compressed_layer"] / peak, 4),
                     "frac_of_8tbs_nominal": round(main_res["attn_gbs_compressed_layer"] / 8000, 4),
                     "algorithmic_bytes_per_launch":
-                        round(main_res["attn_bytes_per_launch_compressed"]),
+                        int_or_none(main_res["attn_bytes_per_launch_compressed"]),
                 },
             },
             "cpu_baseline": cpu,
