@@ -279,7 +279,10 @@ size_t speechkv_decode_workspace_size(int32_t B, int32_t H_q, int32_t H_kv,
  * q            dev, [B][H_q][d].
  * k_cache, v_cache, cache_off, len: as for speechkv_pool (len read only).
  * out          dev, [B][H_q][d], written.
- * H_q / H_kv   must be 1, 2 or 4; d must be 64 or 128; B <= SPEECHKV_MAX_BATCH.
+ * H_q / H_kv   1 to 8 for bf16 (3 to 8 on tensor cores: warp-level bf16 MMA
+ *              with fp32 accumulation, the weights rounded to bf16 before
+ *              P.V and normalised by the sum of the rounded weights), 1, 2
+ *              or 4 for fp32; d must be 64 or 128; B <= SPEECHKV_MAX_BATCH.
  * w, layer, l0 validated only.
  * grid_ctas    CTAs to launch; 0 = automatic (one per SM times the
  *              kernel's residency).  Results do not depend on it beyond

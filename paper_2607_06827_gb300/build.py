@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libspeechkv.so")
-SOURCES = ["api.cu", "pool.cu", "append.cu", "decode_attn.cu", "prefill_attn.cu"]
+SOURCES = ["api.cu", "pool.cu", "append.cu", "decode_attn.cu", "decode_attn_mma.cu", "prefill_attn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC",
               "-Xptxas", "-v", "-I", INCLUDE, "-I", CSRC]

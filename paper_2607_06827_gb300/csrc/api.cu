@@ -17,7 +17,7 @@ __device__ int speechkv_error_word;
 namespace {
 
 constexpr int kMaxDevices = 64;
-constexpr int kDecodeKinds = 12;  // dtype x d x group
+constexpr int kDecodeKinds = 32;  // dtype x d x group (1..8)
 constexpr int kBatchBuckets = 3;  // occupancy is cached per batch-size bucket
 constexpr int kBatchBucketMax[kBatchBuckets] = {128, 512, SPEECHKV_MAX_BATCH};
 
@@ -65,9 +65,9 @@ bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p
 
 bool valid_dtype(speechkv_dtype dt) { return dt == SPEECHKV_F32 || dt == SPEECHKV_BF16; }
 
+// Index of a supported (dtype, d, group) in the per-device occupancy cache.
 int decode_kind(speechkv_dtype dt, int d, int group) {
-    const int g = group == 1 ? 0 : (group == 2 ? 1 : 2);
-    return (dt == SPEECHKV_BF16 ? 6 : 0) + (d == 128 ? 3 : 0) + g;
+    return (dt == SPEECHKV_BF16 ? 16 : 0) + (d == 128 ? 8 : 0) + (group - 1);
 }
 
 // Automatic decode grid: the SM count times the kernel's residency (which

@@ -197,6 +197,53 @@ __device__ __forceinline__ void load16_pairs(const void *p, float2 (&f)[16 / siz
     }
 }
 
+// ---------------------------------------------------------------------------
+// warp-level tensor-core operations (mma.sync / ldmatrix / movmatrix, PTX ISA
+// "Warp-level matrix instructions"); fragment layouts are those of the
+// m16n8k16 shape: lane = 4 r + t holds rows r and r + 8, columns (or k
+// indices) 2t and 2t + 1 (+ 8)
+// ---------------------------------------------------------------------------
+// d += a (16 x 16, row-major fragments) * b (16 x 8, column-major), bf16 in,
+// fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, "
+        "{%4, %5, %6, %7}, {%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Four 8x8 b16 matrices from shared memory; lanes 8i .. 8i + 7 give the row
+// addresses (16 bytes each) of matrix i.  Lane 4r + t receives row r,
+// elements 2t and 2t + 1 of each (transposed: row 2t and 2t + 1, element r).
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr)
+                 : "memory");
+}
+
+// Transpose of an 8x8 b16 matrix held one row pair per lane (lane 4r + t:
+// row r, elements 2t, 2t + 1) into the same layout.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+    uint32_t y;
+    asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
+// Two floats rounded to bf16 (to nearest even) in one word: lo in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
 // Atomic add with acquire-release semantics at GPU scope (publishes the
 // CTA's earlier writes, ordered before it by a barrier, to the acquirer).
 __device__ __forceinline__ int atomic_add_acq_rel_gpu(int *p, int v) {

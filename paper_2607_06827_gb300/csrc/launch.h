@@ -90,6 +90,12 @@ struct DecodeArgs {
 
 // Whether (dtype, d, group) has a compiled decode kernel.
 bool decode_supported(speechkv_dtype dtype, int d, int group);
+// Most query heads per KV head of the bf16 decode instances (tensor-core
+// consumers: the heads of a group are padded to one 8-column MMA tile).
+constexpr int kMmaMaxGroup = 8;
+// The bf16, d = 128 instances (decode_attn_mma.cu).
+int decode_ctas_per_sm_mma128(int group, int B);
+cudaError_t launch_decode_mma128(const DecodeArgs &a, int grid, cudaStream_t stream);
 // Resident CTAs per SM of that kernel on the current device for a batch of
 // B requests (0 on error).
 int decode_ctas_per_sm(speechkv_dtype dtype, int d, int group, int B);

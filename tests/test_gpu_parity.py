@@ -172,6 +172,14 @@ ATTN_CASES = [
     ("f32", 64, 16, 4, (2,), (33,), (1,), (0,), 2),
     ("bf16", 128, 6, 3, (0, 2), (200, 50), (10, 4), (3, 0), 4),  # odd H_kv, group 2
     ("bf16", 64, 5, 5, (0,), (120,), (6,), (1,), 4),              # H_kv = 5, group 1
+    # tensor-core consumers: 3 to 8 query heads per KV head
+    ("bf16", 128, 32, 4, (0, 3), (700, 90), (20, 5), (7, 0), 4),  # group 8
+    ("bf16", 64, 32, 4, (0, 0, 4), (63, 1500, 0), (16, 256, 9), (0, 512, 3), 4),  # group 8
+    ("bf16", 128, 28, 4, (0, 0), (1200, 31), (40, 2), (5, 1), 4),  # group 7
+    ("bf16", 64, 12, 2, (2,), (333,), (7,), (0,), 2),             # group 6
+    ("bf16", 128, 20, 4, (1,), (257,), (4,), (0,), 4),            # group 5
+    ("bf16", 128, 32, 8, (0,), (500,), (20,), (3,), 1),           # group 4
+    ("bf16", 64, 24, 8, (0, 5), (129, 2), (9, 0), (2, 0), 4),     # group 3
 ]
 
 
@@ -276,7 +284,8 @@ def test_invalid_arguments_return_status(sk):
     assert call(w=0) == sk.ERR_INVALID_ARG
     assert call(H_q=7) == sk.ERR_INVALID_ARG
     assert call(d=96) == sk.ERR_UNSUPPORTED
-    assert call(H_q=32, H_kv=4) == sk.ERR_UNSUPPORTED       # group 8 not built
+    assert call(H_q=64, H_kv=4) == sk.ERR_UNSUPPORTED       # group 16 not built
+    assert call(H_q=24, H_kv=8, dt=sk.F32) == sk.ERR_UNSUPPORTED  # fp32: groups 1, 2, 4
     assert call(B=sk.MAX_BATCH + 1) == sk.ERR_UNSUPPORTED
     assert call(wsb=16) == sk.ERR_WORKSPACE
     assert call(grid=-1) == sk.ERR_INVALID_ARG
@@ -362,6 +371,14 @@ def test_fused_step_qwen_and_ragged(sk, oracle):
     _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=4, fused=True)
     wl = inputs.qwen_ragged(B=6)
     _run_steps(sk, oracle, wl, layers=[wl.l0], steps=3, fused=True)
+
+
+@pytest.mark.parametrize("H_q,H_kv", [(32, 4), (28, 4), (24, 8)])
+def test_fused_step_groups_3_to_8(sk, oracle, H_q, H_kv):
+    """Fused steps with the tensor-core consumers (8, 7 and 3 query heads per
+    KV head) on a ragged batch, from the oracle's pooling on."""
+    wl = dataclasses.replace(inputs.qwen_ragged(B=6), H_q=H_q, H_kv=H_kv)
+    _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=3, fused=True)
 
 
 def test_fused_step_matches_separate_calls_and_writes_cache(sk):
@@ -482,6 +499,14 @@ def test_full_size_ragged_sampled(sk, oracle, fused):
     _sampled_full_size(sk, oracle, wl, wl.l0, samples=[0, 17, 64, 127], fused=fused)
 
 
+@pytest.mark.parametrize("H_q,H_kv", [(32, 8), (32, 4), (28, 4)])
+def test_full_size_long_audio_groups(sk, oracle, H_q, H_kv):
+    """The 20 min / w = 4 batch with 4, 8 and 7 query heads per KV head
+    (tensor-core consumers), fused step, sampled requests."""
+    wl = dataclasses.replace(inputs.qwen_long_audio(20, 4, generated=64), H_q=H_q, H_kv=H_kv)
+    _sampled_full_size(sk, oracle, wl, wl.l0, samples=[1, 6], fused=True)
+
+
 def test_full_size_long_audio_fused(sk, oracle):
     wl = inputs.qwen_long_audio(20, 4, generated=64)
     _sampled_full_size(sk, oracle, wl, wl.l0, samples=[3], fused=True)
@@ -517,7 +542,8 @@ def test_max_batch_fused_step(sk, oracle):
         H.assert_close(H.f64(out[b]), ref, "bf16", f"request {b}")
 
 
-@pytest.mark.parametrize("grid,H_kv", [(0, 8), (7, 8), (16, 8), (0, 4), (7, 4), (7, 16)])
+@pytest.mark.parametrize("grid,H_kv", [(0, 8), (7, 8), (16, 8), (0, 4), (7, 4), (7, 16),
+                                     (0, 2), (7, 2)])
 def test_overlap_prior_two_layer_interleave_any_grid(sk, oracle, grid, H_kv):
     """SPEECHKV_OVERLAP_PRIOR with the steps of two layers interleaved
     [a, b, a, b, ...]: the kernel two launches back writes this call's cache
@@ -616,7 +642,8 @@ def test_batch64_30s_pool_and_fused_steps(sk, oracle, w):
     _run_steps(sk, oracle, wl, layers=[wl.l0 - 1, wl.l0], steps=3, fused=True)
 
 
-@pytest.mark.parametrize("H_kv,grid", [(8, 0), (8, 1), (8, 3), (4, 0), (4, 5), (16, 0), (16, 2)])
+@pytest.mark.parametrize("H_kv,grid", [(8, 0), (8, 1), (8, 3), (4, 0), (4, 5), (16, 0), (16, 2),
+                                     (2, 0), (2, 3)])
 def test_short_requests_share_tiles(sk, oracle, H_kv, grid):
     """Many short requests (0-20 rows, some empty) so that a 128-row tile
     holds the ends and starts of several (request, KV head) runs: tiles are
