@@ -53,7 +53,7 @@ L2_FLUSH_BYTES = 256 << 20  # read before each isolated launch (L2 is 129 MB)
 POOL_BATCH = 5  # back-to-back speechkv_pool launches per timed group (setup of each layer)
 PROFILE_TRAFFIC = os.path.join(ROOT, "profiles", "decode_attn_traffic.txt")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2607_06827_gb300", "csrc", f)
-                  for f in ("decode_attn.cu", "common.cuh")]
+                  for f in ("decode_attn.cuh", "decode_attn_mma.cu", "common.cuh")]
 
 
 def parse_args():
@@ -1225,7 +1225,8 @@ def main():
                 "bound": "hbm", "achieved": round(ach, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(ach / peak, 4), "peak_kind": peak_kind,
                 "traffic": profiled_traffic(main_res),
-                "kernel": ("decode_attn_kernel (fused append, bf16, d=128, group 2) of "
+                "kernel": ("decode_attn_kernel (fused append, bf16, d=128, group 2, tensor-core "
+                           "consumers) of "
                            "speechkv_decode_step: the only kernel of the step"),
                 "achieved_from": "algorithmic bytes of all launches of the timed steps / "
                                  "timed-region time (all 28 layers, launch gaps included)",
