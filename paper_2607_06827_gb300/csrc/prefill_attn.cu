@@ -532,10 +532,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int i = 0; i < kBN; i++)
                         if (i > vis) v[i] = __float_as_uint(-INFINITY);
                 }
+                // row maximum: four chains of three-input maxima
                 float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-                for (int i = 0; i < kBN; i++) m4[i & 3] = fmaxf(m4[i & 3], __uint_as_float(v[i]));
-                float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+                for (int i = 0; i < kBN; i += 2)
+                    m4[(i >> 1) & 3] = fmax3(m4[(i >> 1) & 3], __uint_as_float(v[i]),
+                                             __uint_as_float(v[i + 1]));
+                float mx = fmax3(m4[0], m4[1], fmaxf(m4[2], m4[3]));
                 mx *= sl2;
                 // Lazy rescaling: the weights keep using the running maximum
                 // unless the tile's exceeds it by more than 8 (weights then
@@ -543,15 +546,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool bump = mx > m + 8.f;  // always on the first tile (m = -inf)
                 const float mu = bump ? mx : m;
                 const float corr = fast_exp2(m - mu);  // 1 without a bump, 0 on the first tile
-                float sums[4] = {0.f, 0.f, 0.f, 0.f};
+                // exponent arguments and row sums on column pairs (f32x2)
+                const float2 sc2 = make_float2(sl2, sl2), nm2 = make_float2(-mu, -mu);
+                float2 sums[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
                 uint32_t pk[64];
 #pragma unroll
                 for (int i = 0; i < kBN; i += 2) {
-                    const float p0 = fast_exp2(fmaf(__uint_as_float(v[i]), sl2, -mu));
-                    const float p1 = fast_exp2(fmaf(__uint_as_float(v[i + 1]), sl2, -mu));
-                    sums[(i >> 1) & 3] += p0 + p1;
-                    __nv_bfloat162 h = __floats2bfloat162_rn(p0, p1);
-                    pk[i / 2] = *reinterpret_cast<uint32_t *>(&h);
+                    const float2 e = ffma2(make_float2(__uint_as_float(v[i]), __uint_as_float(v[i + 1])),
+                                           sc2, nm2);
+                    const float p0 = fast_exp2(e.x), p1 = fast_exp2(e.y);
+                    sums[(i >> 1) & 1] = fadd2(sums[(i >> 1) & 1], make_float2(p0, p1));
+                    pk[i / 2] = pack_bf16x2(p0, p1);
                 }
                 // P over the first half of S's columns (S is in registers; the
                 // P V that read the previous P completed before this Q K^T)
@@ -567,7 +572,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_st128(tO, o);
                     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                 }
-                l = l * corr + ((sums[0] + sums[1]) + (sums[2] + sums[3]));
+                l = l * corr + ((sums[0].x + sums[1].x) + (sums[0].y + sums[1].y));
                 m = mu;
                 if (x == 0 && e0 + kBN > c) {
                     // value rows at or past the compressed length: zero them
