@@ -115,6 +115,24 @@ __device__ __forceinline__ int64_t pi_of(const Req &q, int64_t t, int w) {
     return t - q.T + q.n;
 }
 
+// packed fp32 pair addition (sm_100+ f32x2) and a three-input maximum
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+// Largest of three floats in one instruction (sm_100+).
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 // ---------------------------------------------------------------- tcgen05 --
 // Shared-memory matrix descriptor, 128-byte swizzle: start address, leading
 // and stride byte offsets (16-byte units), descriptor version 1.
