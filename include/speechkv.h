@@ -211,7 +211,7 @@ speechkv_status speechkv_pool_hidden(const void *h_full,
  *             written for every t < S_b (other rows are left as they are).
  * scale       0 for 1/sqrt(d), else the logit scale.
  * w, layer, l0  w_eff = (layer >= l0 ? w : 1).
- * Supported: SPEECHKV_BF16, d = 128, B <= SPEECHKV_MAX_BATCH, H_q <= 256,
+ * Supported: SPEECHKV_BF16, d = 64 or 128, B <= SPEECHKV_MAX_BATCH, H_q <= 256,
  * q_rows and cache_rows * H_kv below 2^31 (SPEECHKV_ERR_UNSUPPORTED
  * otherwise).  On the device a request whose query rows do not match P+T+N
  * (or lie outside q_rows / cache_rows) sets SPEECHKV_ERR_INVALID_ARG, one

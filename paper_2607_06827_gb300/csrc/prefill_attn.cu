@@ -45,28 +45,37 @@ namespace {
 
 constexpr int kBM = 128;  // query rows per tile = TMEM lanes
 constexpr int kBN = 128;  // keys per tile
-constexpr int kD = 128;   // head dimension
 constexpr int kSlots = 2;    // query tiles per CTA (two query heads of one KV head)
 constexpr int kThreads = 64 + kSlots * 128;  // TMA warp, MMA warp, a softmax warpgroup per slot
-constexpr int kTileBytes = kBM * kD * 2;  // one bf16 tile of 128 rows x 128
-constexpr int kHalf = kTileBytes / 2;     // its 64-column block (128-byte rows)
-constexpr int kKStages = 3;               // key ring
-constexpr int kVStages = 2;               // value ring
-constexpr uint32_t kTmemCols = 512;       // S_x: 128 x, O_x: 256 + 128 x; P_x over S_x's first 64
+constexpr int kBlockBytes = kBM * 128;    // a 64-column block of a tile (128-byte rows)
+constexpr uint32_t kTmemCols = 512;       // S_x: 128 x, O_x: 256 + D x; P_x over S_x's first 64
 
-// shared memory (offsets from a 1024-byte aligned base)
-constexpr int kOffQ = 0;
-constexpr int kOffK = kOffQ + kSlots * kTileBytes;
-constexpr int kOffV = kOffK + kKStages * kTileBytes;
-constexpr int kOffBar = kOffV + kVStages * kTileBytes;
-enum Bar { kQFull, kQEmpty = kQFull + kSlots, kKFull = kQEmpty + kSlots,
-           kKEmpty = kKFull + kKStages, kVFull = kKEmpty + kKStages,
-           kVEmpty = kVFull + kVStages,
-           kSFull = kVEmpty + kVStages,  // [slot]: S_x = Q_x K^T is in TMEM
-           kPFull = kSFull + kSlots,     // [slot]: P_x is in TMEM (the slot's 128 threads)
-           kODone = kPFull + kSlots,     // [slot]: O_x += P_x V is done
-           kDrain = kODone + kSlots, kNumBars };
-constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem address, abort flag, largest tile count
+// Per head dimension D (64 or 128): a tile of 128 rows x D is D / 64 blocks;
+// shared memory (offsets from a 1024-byte aligned base) holds the two query
+// tiles and the key and value rings, then the barriers.
+template <int D>
+struct PfCfg {
+    static constexpr int kTile = kBM * D * 2;
+    static constexpr int kBlocks = D / 64;
+    static constexpr int kKStages = D == 64 ? 5 : 3;  // key ring
+    static constexpr int kVStages = D == 64 ? 4 : 2;  // value ring
+    static constexpr int kOffQ = 0;
+    static constexpr int kOffK = kOffQ + kSlots * kTile;
+    static constexpr int kOffV = kOffK + kKStages * kTile;
+    static constexpr int kOffBar = kOffV + kVStages * kTile;
+    // barriers
+    static constexpr int kQFull = 0, kQEmpty = kQFull + kSlots, kKFull = kQEmpty + kSlots,
+                         kKEmpty = kKFull + kKStages, kVFull = kKEmpty + kKStages,
+                         kVEmpty = kVFull + kVStages,
+                         kSFull = kVEmpty + kVStages,  // [slot]: S_x = Q_x K^T is in TMEM
+                         kPFull = kSFull + kSlots,  // [slot]: P_x is in TMEM (the slot's 128 threads)
+                         kODone = kPFull + kSlots,  // [slot]: O_x += P_x V is done
+                         kDrain = kODone + kSlots, kNumBars = kDrain + 1;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;  // tmem address, abort flag, tile count
+    static constexpr size_t kSmemBytes = (size_t)kOffMisc + 16 + 1024;  // + alignment of the base
+    static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
+    static_assert(D == 64 || D == 128, "head dimension");
+};
 
 struct Req {         // one request's geometry, from the argument arrays
     int64_t q0;      // first query row
@@ -75,8 +84,6 @@ struct Req {         // one request's geometry, from the argument arrays
     int32_t P, T, N, n, S, tiles;
 };
 
-constexpr size_t kSmemBytes = (size_t)kOffMisc + 16 + 1024;  // + alignment of the base
-static_assert(kSmemBytes <= 227 * 1024, "shared memory of one CTA");
 
 // Request b's table entry, read from the argument arrays (cached in L1);
 // tiles = 0 marks a request that is skipped.  *bad: 1 inconsistent, 2 the
@@ -141,10 +148,10 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t addr, uint32_t lbo, uint3
            ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
 }
 // Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, A
-// K-major, B K-major or MN-major, M = 128, N = 128.
-__device__ __forceinline__ uint32_t instr_desc(bool b_mn_major) {
+// K-major, B K-major or MN-major, M = 128, N = n.
+__device__ __forceinline__ uint32_t instr_desc(bool b_mn_major, int n) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
-           ((uint32_t)(kBN >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
+           ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
 }
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
                                      uint32_t accumulate) {
@@ -197,6 +204,29 @@ __device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&r)[64
         :: "r"(taddr), "r"(r[0]),"r"(r[1]),"r"(r[2]),"r"(r[3]),"r"(r[4]),"r"(r[5]),"r"(r[6]),"r"(r[7]),"r"(r[8]),"r"(r[9]),"r"(r[10]),"r"(r[11]),"r"(r[12]),"r"(r[13]),"r"(r[14]),"r"(r[15]),"r"(r[16]),"r"(r[17]),"r"(r[18]),"r"(r[19]),"r"(r[20]),"r"(r[21]),"r"(r[22]),"r"(r[23]),"r"(r[24]),"r"(r[25]),"r"(r[26]),"r"(r[27]),"r"(r[28]),"r"(r[29]),"r"(r[30]),"r"(r[31]),"r"(r[32]),"r"(r[33]),"r"(r[34]),"r"(r[35]),"r"(r[36]),"r"(r[37]),"r"(r[38]),"r"(r[39]),"r"(r[40]),"r"(r[41]),"r"(r[42]),"r"(r[43]),"r"(r[44]),"r"(r[45]),"r"(r[46]),"r"(r[47]),"r"(r[48]),"r"(r[49]),"r"(r[50]),"r"(r[51]),"r"(r[52]),"r"(r[53]),"r"(r[54]),"r"(r[55]),"r"(r[56]),"r"(r[57]),"r"(r[58]),"r"(r[59]),"r"(r[60]),"r"(r[61]),"r"(r[62]),"r"(r[63])
         : "memory");
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 64 fp32 columns of this thread's TMEM lane in one load.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&r)[64]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,%61,%62,%63}, [%64];"
+        : "=r"(r[0]),"=r"(r[1]),"=r"(r[2]),"=r"(r[3]),"=r"(r[4]),"=r"(r[5]),"=r"(r[6]),"=r"(r[7]),"=r"(r[8]),"=r"(r[9]),"=r"(r[10]),"=r"(r[11]),"=r"(r[12]),"=r"(r[13]),"=r"(r[14]),"=r"(r[15]),"=r"(r[16]),"=r"(r[17]),"=r"(r[18]),"=r"(r[19]),"=r"(r[20]),"=r"(r[21]),"=r"(r[22]),"=r"(r[23]),"=r"(r[24]),"=r"(r[25]),"=r"(r[26]),"=r"(r[27]),"=r"(r[28]),"=r"(r[29]),"=r"(r[30]),"=r"(r[31]),"=r"(r[32]),"=r"(r[33]),"=r"(r[34]),"=r"(r[35]),"=r"(r[36]),"=r"(r[37]),"=r"(r[38]),"=r"(r[39]),"=r"(r[40]),"=r"(r[41]),"=r"(r[42]),"=r"(r[43]),"=r"(r[44]),"=r"(r[45]),"=r"(r[46]),"=r"(r[47]),"=r"(r[48]),"=r"(r[49]),"=r"(r[50]),"=r"(r[51]),"=r"(r[52]),"=r"(r[53]),"=r"(r[54]),"=r"(r[55]),"=r"(r[56]),"=r"(r[57]),"=r"(r[58]),"=r"(r[59]),"=r"(r[60]),"=r"(r[61]),"=r"(r[62]),"=r"(r[63])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+// D fp32 columns (64 or 128) of this thread's TMEM lane: load, store.
+template <int N>
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t (&r)[N]) {
+    if constexpr (N == 128) tmem_ld128(taddr, r); else tmem_ld64(taddr, r);
+}
+template <int N>
+__device__ __forceinline__ void tmem_st_cols(uint32_t taddr, const uint32_t (&r)[N]) {
+    if constexpr (N == 128) {
+        tmem_st128(taddr, r);
+        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+    } else {
+        tmem_st64(taddr, r);  // (waits for the store)
+    }
 }
 
 // TMA tensor copies global -> shared (completion as transaction bytes on bar)
@@ -261,6 +291,7 @@ __device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int H_q, int H
     return it;
 }
 
+template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                         const __grid_constant__ CUtensorMap tm_k,
@@ -270,13 +301,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int64_t *__restrict__ cache_off, __nv_bfloat16 *__restrict__ out,
                         int64_t q_rows, int64_t cache_rows, float sl2, int B, int H_q,
                         int H_kv, int w, int *__restrict__ err) {
+    using C = PfCfg<D>;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + kOffBar);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + kOffMisc);
-    volatile int *abort = reinterpret_cast<volatile int *>(sm + kOffMisc + 4);
-    int *tiles_max_s = reinterpret_cast<int *>(sm + kOffMisc + 8);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + C::kOffBar);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + C::kOffMisc);
+    volatile int *abort = reinterpret_cast<volatile int *>(sm + C::kOffMisc + 4);
+    int *tiles_max_s = reinterpret_cast<int *>(sm + C::kOffMisc + 8);
     const ReqSrc tab{q_off, cache_off, Pa, Ta, Na, q_rows, cache_rows, w};
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = H_q / H_kv;
@@ -284,21 +316,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- prologue: barriers, TMEM, largest tile count
     if (tid == 0) {
         for (int x = 0; x < kSlots; x++) {
-            mbar_init(&bar[kQFull + x], 1);
-            mbar_init(&bar[kQEmpty + x], 1);
-            mbar_init(&bar[kSFull + x], 1);
-            mbar_init(&bar[kPFull + x], kBM);
-            mbar_init(&bar[kODone + x], 1);
+            mbar_init(&bar[C::kQFull + x], 1);
+            mbar_init(&bar[C::kQEmpty + x], 1);
+            mbar_init(&bar[C::kSFull + x], 1);
+            mbar_init(&bar[C::kPFull + x], kBM);
+            mbar_init(&bar[C::kODone + x], 1);
         }
-        for (int s = 0; s < kKStages; s++) {
-            mbar_init(&bar[kKFull + s], 1);
-            mbar_init(&bar[kKEmpty + s], 1);
+        for (int s = 0; s < C::kKStages; s++) {
+            mbar_init(&bar[C::kKFull + s], 1);
+            mbar_init(&bar[C::kKEmpty + s], 1);
         }
-        for (int s = 0; s < kVStages; s++) {
-            mbar_init(&bar[kVFull + s], 1);
-            mbar_init(&bar[kVEmpty + s], 1);
+        for (int s = 0; s < C::kVStages; s++) {
+            mbar_init(&bar[C::kVFull + s], 1);
+            mbar_init(&bar[C::kVEmpty + s], 1);
         }
-        mbar_init(&bar[kDrain], 1);
+        mbar_init(&bar[C::kDrain], 1);
         fence_mbar_init();
         *abort = 0;
     }
@@ -329,7 +361,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int tiles_max = *tiles_max_s;
     const int ng = (G + kSlots - 1) / kSlots;
     const int64_t total = (int64_t)tiles_max * B * H_kv * ng;
-    unsigned char *sQ = sm + kOffQ, *sK = sm + kOffK, *sV = sm + kOffV;
+    unsigned char *sQ = sm + C::kOffQ, *sK = sm + C::kOffK, *sV = sm + C::kOffV;
 
     if (warp == 0) {
         // ===================== TMA producer =====================
@@ -342,13 +374,15 @@ __global__ void __launch_bounds__(kThreads, 1)
             int pend_y = -1;                          // cache row of the value tile still to issue
             bool stop = false;
             auto issue_v = [&](int y) -> bool {
-                const int s = (int)(gv % kVStages);
-                const int64_t u = gv / kVStages;
-                if (gv >= kVStages && !wait_bar(&bar[kVEmpty + s], (uint32_t)((u - 1) & 1), abort, err))
+                const int s = (int)(gv % C::kVStages);
+                const int64_t u = gv / C::kVStages;
+                if (gv >= C::kVStages && !wait_bar(&bar[C::kVEmpty + s], (uint32_t)((u - 1) & 1), abort, err))
                     return false;
-                mbar_arrive_expect_tx(&bar[kVFull + s], kTileBytes);
-                tma_2d(sV + s * kTileBytes, &tm_v, 0, y, &bar[kVFull + s]);
-                tma_2d(sV + s * kTileBytes + kHalf, &tm_v, 64, y, &bar[kVFull + s]);
+                mbar_arrive_expect_tx(&bar[C::kVFull + s], C::kTile);
+#pragma unroll
+                for (int blk = 0; blk < C::kBlocks; blk++)
+                    tma_2d(sV + s * C::kTile + blk * kBlockBytes, &tm_v, 64 * blk, y,
+                           &bar[C::kVFull + s]);
                 ++gv;
                 return true;
             };
@@ -363,29 +397,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int x = 0; x < item.n && !stop; x++) {
                     // slot x's query buffer is free once its last Q K^T is done
                     if (uq[x] > 0 &&
-                        !wait_bar(&bar[kQEmpty + x], (uint32_t)((uq[x] - 1) & 1), abort, err)) {
+                        !wait_bar(&bar[C::kQEmpty + x], (uint32_t)((uq[x] - 1) & 1), abort, err)) {
                         stop = true;
                         break;
                     }
-                    unsigned char *sQx = sQ + x * kTileBytes;
-                    mbar_arrive_expect_tx(&bar[kQFull + x], kTileBytes);
-                    tma_3d(sQx, &tm_q, 0, item.hq0 + x, (int)(q.q0 + t0), &bar[kQFull + x]);
-                    tma_3d(sQx + kHalf, &tm_q, 64, item.hq0 + x, (int)(q.q0 + t0), &bar[kQFull + x]);
+                    unsigned char *sQx = sQ + x * C::kTile;
+                    mbar_arrive_expect_tx(&bar[C::kQFull + x], C::kTile);
+#pragma unroll
+                    for (int blk = 0; blk < C::kBlocks; blk++)
+                        tma_3d(sQx + blk * kBlockBytes, &tm_q, 64 * blk, item.hq0 + x,
+                               (int)(q.q0 + t0), &bar[C::kQFull + x]);
                     ++uq[x];
                 }
                 for (int j = 0; j < n_kt && !stop; j++) {
                     // keys are free once their Q K^T is done, values once their P V is
                     const int y = (int)(kvrow + (int64_t)j * kBN);
-                    const int s = (int)(gk % kKStages);
-                    const int64_t u = gk / kKStages;
-                    if (gk >= kKStages &&
-                        !wait_bar(&bar[kKEmpty + s], (uint32_t)((u - 1) & 1), abort, err)) {
+                    const int s = (int)(gk % C::kKStages);
+                    const int64_t u = gk / C::kKStages;
+                    if (gk >= C::kKStages &&
+                        !wait_bar(&bar[C::kKEmpty + s], (uint32_t)((u - 1) & 1), abort, err)) {
                         stop = true;
                         break;
                     }
-                    mbar_arrive_expect_tx(&bar[kKFull + s], kTileBytes);
-                    tma_2d(sK + s * kTileBytes, &tm_k, 0, y, &bar[kKFull + s]);
-                    tma_2d(sK + s * kTileBytes + kHalf, &tm_k, 64, y, &bar[kKFull + s]);
+                    mbar_arrive_expect_tx(&bar[C::kKFull + s], C::kTile);
+#pragma unroll
+                    for (int blk = 0; blk < C::kBlocks; blk++)
+                        tma_2d(sK + s * C::kTile + blk * kBlockBytes, &tm_k, 64 * blk, y,
+                               &bar[C::kKFull + s]);
                     ++gk;
                     if (pend_y >= 0 && !issue_v(pend_y)) {
                         stop = true;
@@ -401,14 +439,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // let every copy issued land before the CTA may exit
             for (int x = 0; x < kSlots; x++)
                 if (uq[x] > 0)
-                    mbar_wait_bounded(&bar[kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
-            for (int64_t x = gk - kKStages; x < gk; x++)
+                    mbar_wait_bounded(&bar[C::kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
+            for (int64_t x = gk - C::kKStages; x < gk; x++)
                 if (x >= 0)
-                    mbar_wait_bounded(&bar[kKFull + (int)(x % kKStages)], (uint32_t)((x / kKStages) & 1),
+                    mbar_wait_bounded(&bar[C::kKFull + (int)(x % C::kKStages)], (uint32_t)((x / C::kKStages) & 1),
                                       err);
-            for (int64_t x = gv - kVStages; x < gv; x++)
+            for (int64_t x = gv - C::kVStages; x < gv; x++)
                 if (x >= 0)
-                    mbar_wait_bounded(&bar[kVFull + (int)(x % kVStages)], (uint32_t)((x / kVStages) & 1),
+                    mbar_wait_bounded(&bar[C::kVFull + (int)(x % C::kVStages)], (uint32_t)((x / C::kVStages) & 1),
                                       err);
         }
     } else if (warp == 1) {
@@ -420,32 +458,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         // the tensor pipe busy meanwhile, and each slot's softmax overlaps
         // the other slot's products.
         if (lane == 0) {
-            const uint32_t id_qk = instr_desc(false), id_pv = instr_desc(true);
+            const uint32_t id_qk = instr_desc(false, kBN), id_pv = instr_desc(true, D);
             const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV);
             // Descriptors are built once per buffer; a K step or a stage only
             // moves the start address, whose field (address / 16, 14 bits)
             // cannot carry over inside shared memory.
             const uint64_t dQ = smem_desc(aQ, 16, 1024);
-            const uint64_t dK = smem_desc(aK, 16, 1024), dV = smem_desc(aV, kHalf, 1024);
-            constexpr uint64_t kStageD = kTileBytes >> 4;
+            const uint64_t dK = smem_desc(aK, 16, 1024), dV = smem_desc(aV, kBlockBytes, 1024);
+            constexpr uint64_t kStageD = C::kTile >> 4;
             int64_t g = 0;                       // key/value tiles
             int64_t ut[kSlots] = {}, uq[kSlots] = {};  // per slot: tiles (P V issued), items
             bool issued = false, stop = false;
             auto qk = [&](int x, int64_t gg) -> bool {  // S_x = Q_x K^T of key tile gg
-                const int s = (int)(gg % kKStages);
-                if (x == 0 && !wait_bar(&bar[kKFull + s], (uint32_t)((gg / kKStages) & 1), abort, err))
+                const int s = (int)(gg % C::kKStages);
+                if (x == 0 && !wait_bar(&bar[C::kKFull + s], (uint32_t)((gg / C::kKStages) & 1), abort, err))
                     return false;
                 // P V of slot x's previous tile has read P_x (inside S_x)
-                if (ut[x] > 0 && !wait_bar(&bar[kODone + x], (uint32_t)((ut[x] - 1) & 1), abort, err))
+                if (ut[x] > 0 && !wait_bar(&bar[C::kODone + x], (uint32_t)((ut[x] - 1) & 1), abort, err))
                     return false;
                 tc_fence_after();
                 const uint64_t dQx = dQ + (uint64_t)x * kStageD, dKs = dK + (uint64_t)s * kStageD;
 #pragma unroll
-                for (int kk = 0; kk < kD / 16; kk++) {
-                    const uint64_t ko = (uint64_t)(((kk >> 2) * kHalf + (kk & 3) * 32) >> 4);
+                for (int kk = 0; kk < D / 16; kk++) {
+                    const uint64_t ko = (uint64_t)(((kk >> 2) * kBlockBytes + (kk & 3) * 32) >> 4);
                     umma(tmem + x * kBN, dQx + ko, dKs + ko, id_qk, kk > 0 ? 1u : 0u);
                 }
-                umma_commit(&bar[kSFull + x]);
+                umma_commit(&bar[C::kSFull + x]);
                 issued = true;
                 return true;
             };
@@ -458,18 +496,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
                 for (int x = 0; x < n && !stop; x++)
-                    stop = !wait_bar(&bar[kQFull + x], (uint32_t)(uq[x] & 1), abort, err);
+                    stop = !wait_bar(&bar[C::kQFull + x], (uint32_t)(uq[x] & 1), abort, err);
                 for (int x = 0; x < n && !stop; x++) stop = !qk(x, g);
                 if (stop) break;
-                umma_commit(&bar[kKEmpty + (int)(g % kKStages)]);
+                umma_commit(&bar[C::kKEmpty + (int)(g % C::kKStages)]);
                 if (n_kt == 1)
-                    for (int x = 0; x < n; x++) umma_commit(&bar[kQEmpty + x]);
+                    for (int x = 0; x < n; x++) umma_commit(&bar[C::kQEmpty + x]);
                 for (int j = 0; j < n_kt && !stop; j++, g++) {
-                    const int sv = (int)(g % kVStages);
+                    const int sv = (int)(g % C::kVStages);
                     for (int x = 0; x < n; x++) {
-                        if (!wait_bar(&bar[kPFull + x], (uint32_t)(ut[x] & 1), abort, err) ||
+                        if (!wait_bar(&bar[C::kPFull + x], (uint32_t)(ut[x] & 1), abort, err) ||
                             (x == 0 &&
-                             !wait_bar(&bar[kVFull + sv], (uint32_t)((g / kVStages) & 1), abort, err))) {
+                             !wait_bar(&bar[C::kVFull + sv], (uint32_t)((g / C::kVStages) & 1), abort, err))) {
                             stop = true;
                             break;
                         }
@@ -478,22 +516,22 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                         for (int kk = 0; kk < kBN / 16; kk++) {
                             const uint64_t vo = (uint64_t)((kk * 16 * 128) >> 4);  // 16 keys further
-                            umma_tmem_a(tmem + 2 * kBN + x * kBN, tmem + x * kBN + kk * 8, dVs + vo,
+                            umma_tmem_a(tmem + 2 * kBN + x * D, tmem + x * kBN + kk * 8, dVs + vo,
                                         id_pv, (j == 0 && kk == 0) ? 0u : 1u);
                         }
-                        umma_commit(&bar[kODone + x]);
+                        umma_commit(&bar[C::kODone + x]);
                         ++ut[x];
-                        if (x == n - 1) umma_commit(&bar[kVEmpty + sv]);  // values of tile j are read
+                        if (x == n - 1) umma_commit(&bar[C::kVEmpty + sv]);  // values of tile j are read
                         if (j + 1 < n_kt) {
                             if (!qk(x, g + 1)) {
                                 stop = true;
                                 break;
                             }
                             if (x == n - 1) {
-                                umma_commit(&bar[kKEmpty + (int)((g + 1) % kKStages)]);
+                                umma_commit(&bar[C::kKEmpty + (int)((g + 1) % C::kKStages)]);
                                 // the query tiles are free once the item's last Q K^T is done
                                 if (j + 2 == n_kt)
-                                    for (int y = 0; y < n; y++) umma_commit(&bar[kQEmpty + y]);
+                                    for (int y = 0; y < n; y++) umma_commit(&bar[C::kQEmpty + y]);
                             }
                         }
                     }
@@ -501,8 +539,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int x = 0; x < n; x++) ++uq[x];
             }
             if (issued) {  // every MMA issued has completed before TMEM is freed
-                umma_commit(&bar[kDrain]);
-                mbar_wait_bounded(&bar[kDrain], 0, err);
+                umma_commit(&bar[C::kDrain]);
+                mbar_wait_bounded(&bar[C::kDrain], 0, err);
             }
         }
     } else {
@@ -511,7 +549,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quarter = warp & 3;         // TMEM lanes 32*quarter .. +31
         const int r = quarter * 32 + lane;    // the row of the tile
         const uint32_t lanes = (uint32_t)(quarter * 32) << 16;
-        const uint32_t tS = tmem + lanes + x * kBN, tO = tmem + lanes + 2 * kBN + x * kBN;
+        const uint32_t tS = tmem + lanes + x * kBN, tO = tmem + lanes + 2 * kBN + x * D;
         int64_t ut = 0, g = 0;  // this slot's tiles; key/value tiles of the CTA
         bool stop = false;
         for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
@@ -531,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int64_t lim = pi_of(q, t < q.S ? t : (int64_t)q.S - 1, w);
             float m = -INFINITY, l = 0.f;
             for (int j = 0; j < n_kt; j++, g++, ut++) {
-                if (!__all_sync(0xffffffffu, wait_bar(&bar[kSFull + x], (uint32_t)(ut & 1), abort, err))) {
+                if (!__all_sync(0xffffffffu, wait_bar(&bar[C::kSFull + x], (uint32_t)(ut & 1), abort, err))) {
                     stop = true;
                     break;
                 }
@@ -582,52 +620,52 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (j > 0 && __any_sync(0xffffffffu, bump)) {
                     // rescale O (the earlier tiles' sum: their P V completed
                     // before this tile's Q K^T was issued)
-                    uint32_t o[128];
-                    tmem_ld128(tO, o);
+                    uint32_t o[D];
+                    tmem_ld_cols<D>(tO, o);
 #pragma unroll
-                    for (int i = 0; i < 128; i++)
+                    for (int i = 0; i < D; i++)
                         o[i] = __float_as_uint(__uint_as_float(o[i]) * corr);
-                    tmem_st128(tO, o);
-                    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                    tmem_st_cols<D>(tO, o);
                 }
                 l = l * corr + ((sums[0].x + sums[1].x) + (sums[0].y + sums[1].y));
                 m = mu;
                 if (x == 0 && e0 + kBN > c) {
                     // value rows at or past the compressed length: zero them
                     // (slot 0's P V reads the stage first)
-                    const int s = (int)(g % kVStages);
-                    if (!__all_sync(0xffffffffu, wait_bar(&bar[kVFull + s],
-                                                          (uint32_t)((g / kVStages) & 1), abort,
+                    const int s = (int)(g % C::kVStages);
+                    if (!__all_sync(0xffffffffu, wait_bar(&bar[C::kVFull + s],
+                                                          (uint32_t)((g / C::kVStages) & 1), abort,
                                                           err))) {
                         stop = true;
                         break;
                     }
                     if (e0 + r >= c) {
-                        unsigned char *row = sV + s * kTileBytes + r * 128;
+                        unsigned char *row = sV + s * C::kTile + r * 128;
 #pragma unroll
-                        for (int y = 0; y < 8; y++) {
-                            *reinterpret_cast<uint4 *>(row + y * 16) = make_uint4(0, 0, 0, 0);
-                            *reinterpret_cast<uint4 *>(row + kHalf + y * 16) = make_uint4(0, 0, 0, 0);
-                        }
+                        for (int blk = 0; blk < C::kBlocks; blk++)
+#pragma unroll
+                            for (int y = 0; y < 8; y++)
+                                *reinterpret_cast<uint4 *>(row + blk * kBlockBytes + y * 16) =
+                                    make_uint4(0, 0, 0, 0);
                     }
                     fence_proxy_async_shared();  // the MMA reads these rows
                 }
                 tc_fence_before();
-                mbar_arrive(&bar[kPFull + x]);
+                mbar_arrive(&bar[C::kPFull + x]);
             }
             if (stop) break;
             // epilogue: O / l once the last P V is done
-            if (!__all_sync(0xffffffffu, wait_bar(&bar[kODone + x], (uint32_t)((ut - 1) & 1), abort,
+            if (!__all_sync(0xffffffffu, wait_bar(&bar[C::kODone + x], (uint32_t)((ut - 1) & 1), abort,
                                                   err)))
                 break;
             tc_fence_after();
             const float inv = 1.f / l;
-            __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq0 + x) * kD;
-            uint32_t o[128];
-            tmem_ld128(tO, o);
+            __nv_bfloat16 *dst = out + ((q.q0 + t) * H_q + item.hq0 + x) * D;
+            uint32_t o[D];
+            tmem_ld_cols<D>(tO, o);
             if (t < q.S) {
 #pragma unroll
-                for (int y = 0; y < 16; y++) {
+                for (int y = 0; y < D / 8; y++) {
                     uint32_t wv[4];
 #pragma unroll
                     for (int z = 0; z < 4; z++) {
@@ -683,40 +721,54 @@ bool encode(CUtensorMap *m, const void *base, int rank, const cuuint64_t *dims,
 
 }  // namespace
 
-bool prefill_supported(speechkv_dtype dtype, int d) { return dtype == SPEECHKV_BF16 && d == kD; }
+namespace {
 
-cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t stream) {
+template <int D>
+cudaError_t launch_prefill_d(const PrefillArgs &a, int num_sms, cudaStream_t stream) {
+    using C = PfCfg<D>;
     CUtensorMap tq, tk, tv;
     {
-        const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.H_q, (cuuint64_t)a.q_rows};
-        const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.H_q * kD * 2};
+        const cuuint64_t dims[3] = {(cuuint64_t)D, (cuuint64_t)a.H_q, (cuuint64_t)a.q_rows};
+        const cuuint64_t strides[2] = {(cuuint64_t)D * 2, (cuuint64_t)a.H_q * D * 2};
         const cuuint32_t box[3] = {64, 1, kBM};
         if (!encode(&tq, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
     }
     {
-        const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)(a.cache_rows * a.H_kv)};
-        const cuuint64_t strides[1] = {(cuuint64_t)kD * 2};
+        const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)(a.cache_rows * a.H_kv)};
+        const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
         const cuuint32_t box[2] = {64, kBN};
         if (!encode(&tk, a.k_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
         if (!encode(&tv, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
     }
-    const size_t smem = kSmemBytes;
+    auto kern = prefill_attn_kernel<D>;
     // the shared-memory opt-in is per device: set it once on each
     static int configured_device_mask = 0;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (!(dev < 31 && (__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev)))) {
-        e = cudaFuncSetAttribute(prefill_attn_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kSmemBytes);
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)C::kSmemBytes);
         if (e != cudaSuccess) return e;
         if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
     }
     const float sl2 = a.scale * 1.4426950408889634f;
-    prefill_attn_kernel<<<num_sms, kThreads, smem, stream>>>(
+    kern<<<num_sms, kThreads, C::kSmemBytes, stream>>>(
         tq, tk, tv, a.q_off, a.P, a.T, a.N, a.cache_off, static_cast<__nv_bfloat16 *>(a.out),
         a.q_rows, a.cache_rows, sl2, a.B, a.H_q, a.H_kv, a.w_eff, a.err);
     return cudaGetLastError();
+}
+
+}  // namespace
+
+bool prefill_supported(speechkv_dtype dtype, int d) {
+    return dtype == SPEECHKV_BF16 && (d == 64 || d == 128);
+}
+
+cudaError_t launch_prefill(const PrefillArgs &a, int num_sms, cudaStream_t stream) {
+    if (a.d == 128) return launch_prefill_d<128>(a, num_sms, stream);
+    if (a.d == 64) return launch_prefill_d<64>(a, num_sms, stream);
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace speechkv

@@ -101,7 +101,7 @@ def test_host_argument_checks_without_gpu():
     pf = lambda B, q_rows, cache_rows, H_q, H_kv, d, w, dt: (  # noqa: E731
         z, z, q_rows, z, z, z, z, z, z, cache_rows, z, 0.0, B, H_q, H_kv, d, w, 0, 0, dt, z)
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.F32)) == sk.ERR_UNSUPPORTED
-    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 64, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 96, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 0, sk.BF16)) == sk.ERR_INVALID_ARG
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 12, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG
     assert lib.speechkv_prefill_attn(*pf(sk.MAX_BATCH + 1, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG

@@ -6,6 +6,8 @@ in the P V product; the bf16 tolerances (max-abs 2e-2, mean-abs 2e-3 on
 unit-variance inputs) apply.  Every case checks the kernel on the GPU's own
 pooled cache (isolating the attention), most also end to end from the same
 full-resolution prompt through the oracle's pooling."""
+import itertools
+
 import numpy as np
 import pytest
 import torch
@@ -16,9 +18,9 @@ from tests import harness as H
 pytestmark = pytest.mark.gpu
 
 
-def _wl(P, T, N, w=4, l0=8, seed=2001, H_q=16, H_kv=8):
+def _wl(P, T, N, w=4, l0=8, seed=2001, H_q=16, H_kv=8, d=128):
     return inputs.Workload(name="prefill", dtype="bf16", L=28, l0=l0, w=w, H_q=H_q, H_kv=H_kv,
-                           d=128, P=list(P), T=list(T), N=list(N), G=[0] * len(T), steps=0,
+                           d=d, P=list(P), T=list(T), N=list(N), G=[0] * len(T), steps=0,
                            seed=seed)
 
 
@@ -68,22 +70,24 @@ def _check(oracle, wl, layer, L, qs, out, full=None):
             H.assert_close(got, ref2, "bf16", f"request {b} end to end")
 
 
-@pytest.mark.parametrize("layer", [8, 0])
-def test_prefill_matches_oracle(oracle, layer):
+@pytest.mark.parametrize("layer,d", [(8, 128), (0, 128), (8, 64), (0, 64)])
+def test_prefill_matches_oracle(oracle, layer, d):
     """A pooled layer (w = 4) and a full-resolution one (causal attention);
-    ragged requests: speech only with text after, a text prefix, text only."""
-    wl = _wl(P=[0, 16, 5], T=[375, 130, 0], N=[32, 7, 40])
+    ragged requests: speech only with text after, a text prefix, text only;
+    head dimensions 128 and 64."""
+    wl = _wl(P=[0, 16, 5], T=[375, 130, 0], N=[32, 7, 40], d=d)
     L, qs, out, full = _run(wl, layer)
     _check(oracle, wl, layer, L, qs, out, full)
 
 
+@pytest.mark.parametrize("d", [128, 64])
 @pytest.mark.parametrize("P,T,N,w", [
     ([0, 0, 0, 3], [1, 128, 512, 1], [0, 0, 1, 0], 4),     # one row, exact tiles, S = 129
     ([0, 7], [255, 1000], [1, 3], 8),                      # w = 8, several key tiles
     ([130, 0], [0, 513], [0, 200], 3),                     # text only; w = 3 (tiles cut windows)
 ])
-def test_prefill_edge_lengths(oracle, P, T, N, w):
-    wl = _wl(P, T, N, w=w, seed=2002)
+def test_prefill_edge_lengths(oracle, P, T, N, w, d):
+    wl = _wl(P, T, N, w=w, seed=2002, d=d)
     L, qs, out, full = _run(wl, 8)
     _check(oracle, wl, 8, L, qs, out, full)
 
@@ -93,8 +97,8 @@ def test_prefill_gqa_groups(oracle):
     work item holds up to two query heads of one KV head: with one head per
     KV head the second tile of every item is idle, with three the items
     alternate between two heads and one."""
-    for H_q, H_kv in ((8, 8), (12, 4), (16, 4)):
-        wl = _wl(P=[4], T=[300], N=[20], H_q=H_q, H_kv=H_kv, seed=2003)
+    for (H_q, H_kv), d in itertools.product(((8, 8), (12, 4), (16, 4)), (128, 64)):
+        wl = _wl(P=[4], T=[300], N=[20], H_q=H_q, H_kv=H_kv, seed=2003, d=d)
         L, qs, out, full = _run(wl, 8)
         _check(oracle, wl, 8, L, qs, out)
 
@@ -206,7 +210,8 @@ def test_prefill_random_shapes(oracle):
         T = [int(x) for x in rng.integers(0, 500, B)]
         N = [max(int(x), 1 if p + t == 0 else 0) for x, p, t in zip(rng.integers(0, 80, B), P, T)]
         layer = int(rng.choice([0, 8]))
-        wl = _wl(P, T, N, w=w, seed=2100 + case, H_q=H_q, H_kv=H_kv)
+        d = int(rng.choice([64, 128]))
+        wl = _wl(P, T, N, w=w, seed=2100 + case, H_q=H_q, H_kv=H_kv, d=d)
         L, full = H.gpu_prefill(wl, layer, extra_rows=int(rng.integers(0, 4)))
         qs = [inputs.prefill_q(wl, layer, b) for b in range(wl.B)]
         q = torch.cat(qs).cuda()
