@@ -384,10 +384,10 @@ speechkv_status speechkv_decode_step_noalloc(
  *              (others may hold anything, e.g. -1).
  * block_size   a power of two; each request's capacity is
  *              max_blocks * block_size rows (at most 2^31 - 1).  The
- *              decode step reads a 128-row tile as one copy per page
- *              segment, the segments issued in parallel: measured against
- *              the contiguous layout, 64-row pages cost 2-4 %, 16-row pages
- *              (vLLM's default) 4-12 %.
+ *              decode step reads a tile in 16-row groups aligned to the
+ *              rows' index (bf16: one copy per group and page, issued in
+ *              parallel): measured against the contiguous layout, 64-row
+ *              pages cost 4-7 %, 16-row pages (vLLM's default) 7-13 %.
  * num_blocks   host: pages in k_pages / v_pages (bounds the table entries).
  * The other arguments, the results and the errors are those of the
  * contiguous entry point of the same name (the rows and their order are the

@@ -253,14 +253,6 @@ __device__ __forceinline__ int atomic_add_acq_rel_gpu(int *p, int v) {
     return old;
 }
 
-// Load with acquire semantics at GPU scope (pairs with release writes of
-// other CTAs: their earlier writes are visible to this thread's later reads).
-__device__ __forceinline__ int ld_acquire_gpu(const int *p) {
-    int v;
-    asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-    return v;
-}
-
 // Hint: bring `bytes` (a multiple of 16, 16-byte aligned) of global memory
 // into L2.  No value is read; later reads see whatever the memory holds then.
 __device__ __forceinline__ void prefetch_l2(const void *p, uint32_t bytes) {

@@ -626,28 +626,25 @@ __global__ void __launch_bounds__(DecodeCfg<T, D, G>::kThreads, DecodeCfg<T, D, 
             if (lane == 0) mbar_arrive(&free_bar[x]);  // the buffer may be refilled
             if (ok && !whole) {
                 // Split piece: the CTA that finishes last at this (request,
-                // head) merges every piece.  First peek at the ticket: when all
-                // the other CTAs have published already, this one is last and
-                // merges straight from its registers.  Otherwise publish this
-                // partial, then take a ticket (acquire-release) to find out.
-                int last = 0;
-                if (lane == 0) last = ld_acquire_gpu(&counters[seg]) == others;
-                last = __shfl_sync(0xffffffffu, last, 0);
-                if (!last) {
-                    float *slot = partials + (c + seg) * slot_floats;  // o [G][D], m [G], l [G]
+                // head) merges every piece.  Publish this partial, then take a
+                // ticket (acquire-release) to find out whether this CTA is the
+                // last; the last one merges with its own state from registers.
+                // (One L2 round trip for the CTAs that only publish: a CTA's
+                // exit frees its SM for the next launch's CTA.)
+                float *slot = partials + (c + seg) * slot_floats;  // o [G][D], m [G], l [G]
 #pragma unroll
-                    for (int g = 0; g < G; g++) {
+                for (int g = 0; g < G; g++) {
 #pragma unroll
-                        for (int i = 0; i < kCols; i++) slot[g * D + lane * kCols + i] = acc[g][i];
-                        if (lane == 0) {
-                            slot[G * D + g] = M[g];
-                            slot[G * D + G + g] = Ls[g];
-                        }
+                    for (int i = 0; i < kCols; i++) slot[g * D + lane * kCols + i] = acc[g][i];
+                    if (lane == 0) {
+                        slot[G * D + g] = M[g];
+                        slot[G * D + G + g] = Ls[g];
                     }
-                    __syncwarp();  // the lanes' partial writes precede lane 0's release
-                    if (lane == 0) last = atomic_add_acq_rel_gpu(&counters[seg], 1) == others;
-                    last = __shfl_sync(0xffffffffu, last, 0);
                 }
+                __syncwarp();  // the lanes' partial writes precede lane 0's release
+                int last = 0;
+                if (lane == 0) last = atomic_add_acq_rel_gpu(&counters[seg], 1) == others;
+                last = __shfl_sync(0xffffffffu, last, 0);
                 __syncwarp();  // lane 0's acquire orders the other lanes' reads too
                 if (last) {
                     // online log-sum-exp over the pieces in CTA order (this
