@@ -550,7 +550,8 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
     layer (l0) and at a full-resolution one (0): CUDA-event time of one launch
     (median of `repeats`), algorithmic FLOPs (4 d per visible query-key pair:
     QK^T and PV) and the fraction of the measured bf16 tensor peak (burst:
-    the kernel is timed alone)."""
+    the kernel is timed alone).  The same cache copied into 16-row pages of a
+    shuffled block table times speechkv_prefill_attn_paged beside it."""
     import numpy as np
     import torch
     from paper_2607_06827_gb300 import inputs, speechkv as sk
@@ -582,30 +583,57 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
             pairs += int((pi + 1).sum())
         flops = 4.0 * wl.d * wl.H_q * pairs
 
-        def launch():
-            sk.prefill_attn(q, q_off, P, T, N, kc, vc, cache_off, out, wl.w, layer, wl.l0,
-                            wl.H_kv)
-        for _ in range(warmup):
-            launch()
-        torch.cuda.synchronize()
-        times = []
-        t0 = time.time()
-        for _ in range(repeats):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record()
-            launch()
-            e1.record()
+        # the same rows in 16-row pages (shuffled block table)
+        bs = PREFILL_PAGE_ROWS
+        need = [-(-c // bs) for c in cap]
+        perm = torch.from_numpy(np.random.default_rng(layer).permutation(sum(need))).cuda()
+        table = torch.full((wl.B, max(need)), -1, dtype=torch.int32, device="cuda")
+        kp = torch.empty((sum(need), wl.H_kv, bs, wl.d), dtype=torch.bfloat16, device="cuda")
+        vp = torch.empty_like(kp)
+        first = 0
+        for b in range(wl.B):
+            ids = perm[first:first + need[b]]
+            first += need[b]
+            table[b, :need[b]] = ids.to(torch.int32)
+            for src, dst in ((kc, kp), (vc, vp)):
+                blk = src[int(coff[b]) * wl.H_kv * wl.d:int(coff[b + 1]) * wl.H_kv * wl.d]
+                blk = blk.view(wl.H_kv, cap[b], wl.d)
+                pad = torch.zeros((wl.H_kv, need[b] * bs, wl.d), dtype=blk.dtype, device="cuda")
+                pad[:, :cap[b]] = blk
+                dst[ids] = pad.view(wl.H_kv, need[b], bs, wl.d).permute(1, 0, 2, 3)
+
+        def launch(paged):
+            if paged:
+                sk.prefill_attn_paged(q, q_off, P, T, N, kp, vp, table, out, wl.w, layer, wl.l0)
+            else:
+                sk.prefill_attn(q, q_off, P, T, N, kc, vc, cache_off, out, wl.w, layer, wl.l0,
+                                wl.H_kv)
+        med = {}
+        for paged in (False, True):
+            for _ in range(warmup):
+                launch(paged)
             torch.cuda.synchronize()
-            times.append(e0.elapsed_time(e1))
-        clocks and clocks.mark(t0, time.time())
-        status = sk.check_device_error()
-        assert status == sk.OK, sk.status_string(status)
-        assert bool(torch.isfinite(out.float()).all())
-        ms = sorted(times)[len(times) // 2]
+            times = []
+            t0 = time.time()
+            for _ in range(repeats):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                launch(paged)
+                e1.record()
+                torch.cuda.synchronize()
+                times.append(e0.elapsed_time(e1))
+            clocks and clocks.mark(t0, time.time())
+            status = sk.check_device_error()
+            assert status == sk.OK, sk.status_string(status)
+            assert bool(torch.isfinite(out.float()).all())
+            med[paged] = sorted(times)[len(times) // 2]
+        ms = med[False]
         res[kind] = {"layer": layer, "w_eff": w_eff, "us": round(ms * 1e3, 1),
                      "tflop": round(flops / 1e12, 4),
-                     "tflops": round(flops / (ms * 1e-3) / 1e12, 1)}
-        del kc, vc
+                     "tflops": round(flops / (ms * 1e-3) / 1e12, 1),
+                     "us_paged": round(med[True] * 1e3, 1),
+                     "paged_over_contiguous": round(med[True] / ms, 4)}
+        del kc, vc, kp, vp
     del q, out
     torch.cuda.empty_cache()
     peak, kind = measured_bf16_peak()
@@ -613,12 +641,14 @@ def measure_prefill(wl, clocks, repeats: int = 5, warmup: int = 2):
         r["frac"] = round(r["tflops"] / peak, 4)
     res["hs_pool"] = measure_hs_pool(wl, clocks, repeats, warmup)
     res.update({"bound": "tensor", "peak": peak, "peak_kind": kind, "unit": "TFLOP/s",
-                "kernel": "prefill_attn_kernel (tcgen05, bf16, d=128): speechkv_prefill_attn",
+                "kernel": ("prefill_attn_kernel (tcgen05, bf16, d=128): speechkv_prefill_attn; "
+                           "us_paged: speechkv_prefill_attn_paged, 16-row pages"),
                 "workload": f"whole prompt of the batch ({S} query rows x {wl.H_q} heads)"})
     return res
 
 
 PAGE_SIZES = (16, 32, 64)  # rows per page of the paged-cache measurement
+PREFILL_PAGE_ROWS = 16     # rows per page of the paged prefill beside the contiguous one
 
 
 def measure_paged(wl, clocks, steps: int = 64, warmup: int = 4, chunk: int = 32):

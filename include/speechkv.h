@@ -424,6 +424,21 @@ speechkv_status speechkv_decode_step_paged(
     int32_t layer, int32_t l0, int32_t grid_ctas, void *workspace,
     size_t workspace_bytes, speechkv_dtype dtype, uint32_t flags,
     cudaStream_t stream);
+/*
+ * speechkv_prefill_attn_paged -- speechkv_prefill_attn over a paged cache
+ * (pages as above; no cache_off / cache_rows).  block_size must be at least 8
+ * (a key tile is copied as one piece per page of whole 8-row swizzle atoms;
+ * SPEECHKV_ERR_UNSUPPORTED below that); num_blocks * H_kv * block_size must
+ * stay below 2^31.  Pages past a request's compressed rows are not read.
+ * Results are bit-identical to speechkv_prefill_attn over the same rows.
+ */
+speechkv_status speechkv_prefill_attn_paged(
+    const void *q, const int64_t *q_off, int64_t q_rows, const int32_t *P,
+    const int32_t *T, const int32_t *N, const void *k_pages,
+    const void *v_pages, const int32_t *block_table, int32_t max_blocks,
+    int32_t block_size, int64_t num_blocks, void *out, float scale,
+    int32_t B, int32_t H_q, int32_t H_kv, int32_t d, int32_t w,
+    int32_t layer, int32_t l0, speechkv_dtype dtype, cudaStream_t stream);
 
 /*
  * Synchronises `stream`, then reads and clears the current device's error

@@ -398,28 +398,36 @@ speechkv_status speechkv_pool_hidden(const void *h_full, const int64_t *full_off
                : SPEECHKV_ERR_CUDA;
 }
 
-speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64_t q_rows,
+// Host checks and launch of speechkv_prefill_attn and its paged form
+// (map.table != nullptr: k_cache / v_cache are the page pools).
+static speechkv_status prefill_common(const void *q, const int64_t *q_off, int64_t q_rows,
                                       const int32_t *P, const int32_t *T, const int32_t *N,
                                       const void *k_cache, const void *v_cache,
                                       const int64_t *cache_off, int64_t cache_rows, void *out,
                                       float scale, int32_t B, int32_t H_q, int32_t H_kv,
                                       int32_t d, int32_t w, int32_t layer, int32_t l0,
-                                      speechkv_dtype dtype, cudaStream_t stream) {
+                                      speechkv_dtype dtype, cudaStream_t stream,
+                                      const speechkv::CacheMap &map) {
+    const bool paged = map.table != nullptr;
     if (B < 0 || B > SPEECHKV_MAX_BATCH || q_rows < 0 || cache_rows < 0 || H_q < 1 ||
         H_kv < 1 || H_q % H_kv != 0 || w < 1 || layer < 0 || l0 < 0 || !valid_dtype(dtype) ||
         isnan(scale) || isinf(scale) || scale < 0.f)
         return SPEECHKV_ERR_INVALID_ARG;
     if (!speechkv::prefill_supported(dtype, d)) return SPEECHKV_ERR_UNSUPPORTED;
-    // tensor-copy coordinates are 32-bit
-    if (q_rows >= (1ll << 31) || cache_rows * (int64_t)H_kv >= (1ll << 31) || H_q > 256)
+    // tensor-copy coordinates are 32-bit; a page is copied as whole 8-row
+    // swizzle atoms
+    const int64_t kv_rows =
+        paged ? map.num_blocks * H_kv * ((int64_t)1 << map.bs_log2) : cache_rows * (int64_t)H_kv;
+    if (q_rows >= (1ll << 31) || kv_rows >= (1ll << 31) || H_q > 256 ||
+        (paged && map.bs_log2 < 3))
         return SPEECHKV_ERR_UNSUPPORTED;
     if (B == 0 || q_rows == 0) return SPEECHKV_OK;
-    if (!q || !q_off || !P || !T || !N || !k_cache || !v_cache || !cache_off || !out ||
-        cache_rows == 0)
+    if (!q || !q_off || !P || !T || !N || !k_cache || !v_cache || (!paged && !cache_off) ||
+        !out || (!paged && cache_rows == 0))
         return SPEECHKV_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(out, 16) ||
-        !aligned(q_off, 8) || !aligned(cache_off, 8) || !aligned(P, 4) || !aligned(T, 4) ||
-        !aligned(N, 4))
+        !aligned(q_off, 8) || (!paged && !aligned(cache_off, 8)) || !aligned(P, 4) ||
+        !aligned(T, 4) || !aligned(N, 4))
         return SPEECHKV_ERR_INVALID_ARG;
     DeviceState *s = nullptr;
     speechkv_status st = device_state(&s);
@@ -433,8 +441,8 @@ speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64
     a.N = N;
     a.k_cache = k_cache;
     a.v_cache = v_cache;
-    a.cache_off = cache_off;
-    a.cache_rows = cache_rows;
+    a.cache_off = paged ? nullptr : cache_off;
+    a.cache_rows = paged ? 0 : cache_rows;
     a.out = out;
     a.scale = scale > 0.f ? scale : 1.f / sqrtf((float)d);
     a.B = B;
@@ -443,8 +451,35 @@ speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64
     a.d = d;
     a.w_eff = layer >= l0 ? w : 1;
     a.err = s->err;
+    a.map = map;
     return speechkv::launch_prefill(a, s->num_sms, stream) == cudaSuccess ? SPEECHKV_OK
                                                                           : SPEECHKV_ERR_CUDA;
+}
+
+speechkv_status speechkv_prefill_attn(const void *q, const int64_t *q_off, int64_t q_rows,
+                                      const int32_t *P, const int32_t *T, const int32_t *N,
+                                      const void *k_cache, const void *v_cache,
+                                      const int64_t *cache_off, int64_t cache_rows, void *out,
+                                      float scale, int32_t B, int32_t H_q, int32_t H_kv,
+                                      int32_t d, int32_t w, int32_t layer, int32_t l0,
+                                      speechkv_dtype dtype, cudaStream_t stream) {
+    return prefill_common(q, q_off, q_rows, P, T, N, k_cache, v_cache, cache_off, cache_rows,
+                          out, scale, B, H_q, H_kv, d, w, layer, l0, dtype, stream,
+                          speechkv::CacheMap{});
+}
+
+speechkv_status speechkv_prefill_attn_paged(
+    const void *q, const int64_t *q_off, int64_t q_rows, const int32_t *P, const int32_t *T,
+    const int32_t *N, const void *k_pages, const void *v_pages, const int32_t *block_table,
+    int32_t max_blocks, int32_t block_size, int64_t num_blocks, void *out, float scale,
+    int32_t B, int32_t H_q, int32_t H_kv, int32_t d, int32_t w, int32_t layer, int32_t l0,
+    speechkv_dtype dtype, cudaStream_t stream) {
+    speechkv::CacheMap m;
+    if (B == 0 || q_rows == 0) return SPEECHKV_OK;
+    const speechkv_status st = make_map(block_table, max_blocks, block_size, num_blocks, &m);
+    if (st != SPEECHKV_OK) return st;
+    return prefill_common(q, q_off, q_rows, P, T, N, k_pages, v_pages, nullptr, 0, out, scale,
+                          B, H_q, H_kv, d, w, layer, l0, dtype, stream, m);
 }
 
 }  // extern "C"

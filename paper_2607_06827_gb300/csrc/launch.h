@@ -115,6 +115,7 @@ struct PrefillArgs {
     float scale;         // > 0
     int32_t B, H_q, H_kv, d, w_eff;
     int *err;
+    CacheMap map;  // paged layout when map.table != nullptr (cache_off, cache_rows unused)
 };
 // Whether (dtype, d) has a compiled prefill kernel.
 bool prefill_supported(speechkv_dtype dtype, int d);

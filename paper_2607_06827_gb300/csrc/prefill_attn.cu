@@ -87,18 +87,21 @@ struct Req {         // one request's geometry, from the argument arrays
 
 // Request b's table entry, read from the argument arrays (cached in L1);
 // tiles = 0 marks a request that is skipped.  *bad: 1 inconsistent, 2 the
-// compressed rows exceed the capacity.
+// compressed rows exceed the capacity.  A paged cache (kPaged; no cache_off)
+// gives every request capP rows.
+template <bool kPaged>
 struct ReqSrc {
     const int64_t *q_off, *cache_off;
     const int32_t *P, *T, *N;
     int64_t q_rows, cache_rows;
     int w;
+    int64_t capP;
     __device__ __forceinline__ Req operator()(int b, int *bad = nullptr) const {
         Req q;
         q.q0 = q_off[b];
         const int64_t q1 = q_off[b + 1];
-        q.kv0 = cache_off[b];
-        const int64_t kv1 = cache_off[b + 1];
+        q.kv0 = kPaged ? 0 : cache_off[b];
+        const int64_t kv1 = kPaged ? capP : cache_off[b + 1];
         q.cap = kv1 - q.kv0;
         q.P = P[b];
         q.T = T[b];
@@ -108,7 +111,8 @@ struct ReqSrc {
         const int64_t c = (int64_t)q.P + q.n + q.N;
         q.S = (int32_t)S;
         const bool ok = q.P >= 0 && q.T >= 0 && q.N >= 0 && q.q0 >= 0 && q1 - q.q0 == S &&
-                        q1 <= q_rows && q.kv0 >= 0 && kv1 <= cache_rows && S < (1ll << 31);
+                        q1 <= q_rows && q.kv0 >= 0 && (kPaged || kv1 <= cache_rows) &&
+                        S < (1ll << 31);
         const int why = !ok ? 1 : (c > q.cap ? 2 : 0);
         if (bad) *bad = why;
         q.tiles = why == 0 ? (int32_t)((S + kBM - 1) / kBM) : 0;
@@ -273,8 +277,9 @@ struct Item {
     int b, hq0, n, i;  // request, first query head, heads (slots used), query tile
     bool valid;
 };
+template <bool kPaged>
 __device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int H_q, int H_kv,
-                                        const ReqSrc &tab, Req &q) {
+                                        const ReqSrc<kPaged> &tab, Req &q) {
     Item it;
     const int G = H_q / H_kv;
     const int ng = (G + kSlots - 1) / kSlots;    // head groups of a KV head
@@ -291,7 +296,9 @@ __device__ __forceinline__ Item item_at(int64_t k, int tiles_max, int H_q, int H
     return it;
 }
 
-template <int D>
+// kPaged: the cache is paged through map's block table (its own instance, so
+// that the contiguous kernel carries none of that code).
+template <int D, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 1)
     prefill_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
                         const __grid_constant__ CUtensorMap tm_k,
@@ -300,7 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int32_t *__restrict__ Ta, const int32_t *__restrict__ Na,
                         const int64_t *__restrict__ cache_off, __nv_bfloat16 *__restrict__ out,
                         int64_t q_rows, int64_t cache_rows, float sl2, int B, int H_q,
-                        int H_kv, int w, int *__restrict__ err) {
+                        int H_kv, int w, int *__restrict__ err, CacheMap map) {
     using C = PfCfg<D>;
     extern __shared__ unsigned char smem_raw[];
     unsigned char *sm = reinterpret_cast<unsigned char *>(
@@ -309,7 +316,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(sm + C::kOffMisc);
     volatile int *abort = reinterpret_cast<volatile int *>(sm + C::kOffMisc + 4);
     int *tiles_max_s = reinterpret_cast<int *>(sm + C::kOffMisc + 8);
-    const ReqSrc tab{q_off, cache_off, Pa, Ta, Na, q_rows, cache_rows, w};
+    const ReqSrc<kPaged> tab{q_off,      cache_off, Pa, Ta, Na, q_rows,
+                             cache_rows, w,         (int64_t)map.max_blocks << map.bs_log2};
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int G = H_q / H_kv;
 
@@ -369,85 +377,198 @@ __global__ void __launch_bounds__(kThreads, 1)
         // item (one buffer per slot), then its key and value tiles with the
         // keys one tile ahead of the values (a value tile waits for an older
         // P V than the key tile issued before it).
-        if (lane == 0) {
-            int64_t uq[kSlots] = {}, gk = 0, gv = 0;  // query (per slot), key, value tiles issued
-            int pend_y = -1;                          // cache row of the value tile still to issue
-            bool stop = false;
-            auto issue_v = [&](int y) -> bool {
-                const int s = (int)(gv % C::kVStages);
-                const int64_t u = gv / C::kVStages;
-                if (gv >= C::kVStages && !wait_bar(&bar[C::kVEmpty + s], (uint32_t)((u - 1) & 1), abort, err))
-                    return false;
-                mbar_arrive_expect_tx(&bar[C::kVFull + s], C::kTile);
+        if constexpr (!kPaged) {
+            if (lane == 0) {
+                int64_t uq[kSlots] = {}, gk = 0, gv = 0;  // query (per slot), key, value tiles issued
+                int pend_y = -1;                          // cache row of the value tile still to issue
+                bool stop = false;
+                auto issue_v = [&](int y) -> bool {
+                    const int s = (int)(gv % C::kVStages);
+                    const int64_t u = gv / C::kVStages;
+                    if (gv >= C::kVStages && !wait_bar(&bar[C::kVEmpty + s], (uint32_t)((u - 1) & 1), abort, err))
+                        return false;
+                    mbar_arrive_expect_tx(&bar[C::kVFull + s], C::kTile);
 #pragma unroll
-                for (int blk = 0; blk < C::kBlocks; blk++)
-                    tma_2d(sV + s * C::kTile + blk * kBlockBytes, &tm_v, 64 * blk, y,
-                           &bar[C::kVFull + s]);
-                ++gv;
-                return true;
+                    for (int blk = 0; blk < C::kBlocks; blk++)
+                        tma_2d(sV + s * C::kTile + blk * kBlockBytes, &tm_v, 64 * blk, y,
+                               &bar[C::kVFull + s]);
+                    ++gv;
+                    return true;
+                };
+                for (int64_t k = blockIdx.x; k < total && !stop && !*abort; k += gridDim.x) {
+                    Req q;
+                    const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
+                    if (!item.valid) continue;
+                    const int64_t t0 = (int64_t)item.i * kBM;
+                    const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
+                    const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
+                    const int64_t kvrow = q.kv0 * H_kv + (int64_t)(item.hq0 / G) * q.cap;
+                    for (int x = 0; x < item.n && !stop; x++) {
+                        // slot x's query buffer is free once its last Q K^T is done
+                        if (uq[x] > 0 &&
+                            !wait_bar(&bar[C::kQEmpty + x], (uint32_t)((uq[x] - 1) & 1), abort, err)) {
+                            stop = true;
+                            break;
+                        }
+                        unsigned char *sQx = sQ + x * C::kTile;
+                        mbar_arrive_expect_tx(&bar[C::kQFull + x], C::kTile);
+#pragma unroll
+                        for (int blk = 0; blk < C::kBlocks; blk++)
+                            tma_3d(sQx + blk * kBlockBytes, &tm_q, 64 * blk, item.hq0 + x,
+                                   (int)(q.q0 + t0), &bar[C::kQFull + x]);
+                        ++uq[x];
+                    }
+                    for (int j = 0; j < n_kt && !stop; j++) {
+                        // keys are free once their Q K^T is done, values once their P V is
+                        const int y = (int)(kvrow + (int64_t)j * kBN);
+                        const int s = (int)(gk % C::kKStages);
+                        const int64_t u = gk / C::kKStages;
+                        if (gk >= C::kKStages &&
+                            !wait_bar(&bar[C::kKEmpty + s], (uint32_t)((u - 1) & 1), abort, err)) {
+                            stop = true;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(&bar[C::kKFull + s], C::kTile);
+#pragma unroll
+                        for (int blk = 0; blk < C::kBlocks; blk++)
+                            tma_2d(sK + s * C::kTile + blk * kBlockBytes, &tm_k, 64 * blk, y,
+                                   &bar[C::kKFull + s]);
+                        ++gk;
+                        if (pend_y >= 0 && !issue_v(pend_y)) {
+                            stop = true;
+                            break;
+                        }
+                        pend_y = y;
+                    }
+                    // the item's last value tile now, not behind the next item's
+                    // query-buffer wait (its P V would stall on the load)
+                    if (!stop && pend_y >= 0) stop = !issue_v(pend_y);
+                    pend_y = -1;
+                }
+                // let every copy issued land before the CTA may exit
+                for (int x = 0; x < kSlots; x++)
+                    if (uq[x] > 0)
+                        mbar_wait_bounded(&bar[C::kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
+                for (int64_t x = gk - C::kKStages; x < gk; x++)
+                    if (x >= 0)
+                        mbar_wait_bounded(&bar[C::kKFull + (int)(x % C::kKStages)], (uint32_t)((x / C::kKStages) & 1),
+                                          err);
+                for (int64_t x = gv - C::kVStages; x < gv; x++)
+                    if (x >= 0)
+                        mbar_wait_bounded(&bar[C::kVFull + (int)(x % C::kVStages)], (uint32_t)((x / C::kVStages) & 1),
+                                          err);
+            }
+        } else {
+            // Paged: every lane walks the same items and tiles; lane 0 waits
+            // for the stages, sets the expected bytes and copies the queries,
+            // and lane p copies page p of a key or value tile (pages of 8
+            // rows or more: at most 16 per 128-row tile), so that the small
+            // copies are issued in parallel.  Pages past the compressed rows
+            // are not read (their rows are masked, and the values zeroed, by
+            // the softmax warps).
+            int64_t uq[kSlots] = {}, gk = 0, gv = 0;  // query (per slot), key, value tiles issued
+            int pend = -1;                            // key tile whose values are still to issue
+            bool stop = false;
+            const int lg = map.bs_log2;
+            const int rows = lg < 7 ? 1 << lg : kBN;  // rows per copy (the maps' box)
+            auto wait0 = [&](uint64_t *b, uint32_t parity) -> bool {  // lane 0 waits for all
+                int ok = 1;
+                if (lane == 0) ok = wait_bar(b, parity, abort, err);
+                return __shfl_sync(0xffffffffu, ok, 0) != 0;
             };
-            for (int64_t k = blockIdx.x; k < total && !stop && !*abort; k += gridDim.x) {
+            for (int64_t k = blockIdx.x; k < total && !stop; k += gridDim.x) {
+                if (__shfl_sync(0xffffffffu, lane == 0 ? (int)*abort : 0, 0)) break;
                 Req q;
                 const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
                 if (!item.valid) continue;
                 const int64_t t0 = (int64_t)item.i * kBM;
                 const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
-                const int64_t kvrow = q.kv0 * H_kv + (int64_t)(item.hq0 / G) * q.cap;
+                const int hk = item.hq0 / G;                      // the KV head
+                const int64_t crows = (int64_t)q.P + q.n + q.N;  // compressed rows
+                auto copy_tile = [&](unsigned char *dst, const CUtensorMap *tm, int kt,
+                                     uint64_t *fb) {
+                    const int64_t r0 = (int64_t)kt * kBN;
+                    int ncopy = 0;
+                    while (ncopy < kBN / rows && r0 + (int64_t)ncopy * rows < crows) ncopy++;
+                    if (lane == 0) mbar_arrive_expect_tx(fb, (uint32_t)(ncopy * rows * 128 * C::kBlocks));
+                    __syncwarp();
+                    if (lane < ncopy) {
+                        const int64_t r = r0 + (int64_t)lane * rows;
+                        int32_t blk_id =
+                            __ldg(map.table + (int64_t)item.b * map.max_blocks + (r >> lg));
+                        if (blk_id < 0 || blk_id >= map.num_blocks) {
+                            report_error(err, SPEECHKV_ERR_INVALID_ARG);  // read page 0 instead
+                            blk_id = 0;
+                        }
+                        const int y = (int)((((int64_t)blk_id * H_kv + hk) << lg) +
+                                            (r & ((1ll << lg) - 1)));
+#pragma unroll
+                        for (int blk = 0; blk < C::kBlocks; blk++)
+                            tma_2d(dst + blk * kBlockBytes + lane * rows * 128, tm, 64 * blk, y,
+                                   fb);
+                    }
+                };
+                auto issue_v = [&](int kt) -> bool {
+                    const int s = (int)(gv % C::kVStages);
+                    const int64_t u = gv / C::kVStages;
+                    if (gv >= C::kVStages && !wait0(&bar[C::kVEmpty + s], (uint32_t)((u - 1) & 1)))
+                        return false;
+                    copy_tile(sV + s * C::kTile, &tm_v, kt, &bar[C::kVFull + s]);
+                    ++gv;
+                    return true;
+                };
                 for (int x = 0; x < item.n && !stop; x++) {
                     // slot x's query buffer is free once its last Q K^T is done
-                    if (uq[x] > 0 &&
-                        !wait_bar(&bar[C::kQEmpty + x], (uint32_t)((uq[x] - 1) & 1), abort, err)) {
+                    if (uq[x] > 0 && !wait0(&bar[C::kQEmpty + x], (uint32_t)((uq[x] - 1) & 1))) {
                         stop = true;
                         break;
                     }
-                    unsigned char *sQx = sQ + x * C::kTile;
-                    mbar_arrive_expect_tx(&bar[C::kQFull + x], C::kTile);
+                    if (lane == 0) {
+                        unsigned char *sQx = sQ + x * C::kTile;
+                        mbar_arrive_expect_tx(&bar[C::kQFull + x], C::kTile);
 #pragma unroll
-                    for (int blk = 0; blk < C::kBlocks; blk++)
-                        tma_3d(sQx + blk * kBlockBytes, &tm_q, 64 * blk, item.hq0 + x,
-                               (int)(q.q0 + t0), &bar[C::kQFull + x]);
+                        for (int blk = 0; blk < C::kBlocks; blk++)
+                            tma_3d(sQx + blk * kBlockBytes, &tm_q, 64 * blk, item.hq0 + x,
+                                   (int)(q.q0 + t0), &bar[C::kQFull + x]);
+                    }
                     ++uq[x];
                 }
                 for (int j = 0; j < n_kt && !stop; j++) {
                     // keys are free once their Q K^T is done, values once their P V is
-                    const int y = (int)(kvrow + (int64_t)j * kBN);
                     const int s = (int)(gk % C::kKStages);
                     const int64_t u = gk / C::kKStages;
-                    if (gk >= C::kKStages &&
-                        !wait_bar(&bar[C::kKEmpty + s], (uint32_t)((u - 1) & 1), abort, err)) {
+                    if (gk >= C::kKStages && !wait0(&bar[C::kKEmpty + s], (uint32_t)((u - 1) & 1))) {
                         stop = true;
                         break;
                     }
-                    mbar_arrive_expect_tx(&bar[C::kKFull + s], C::kTile);
-#pragma unroll
-                    for (int blk = 0; blk < C::kBlocks; blk++)
-                        tma_2d(sK + s * C::kTile + blk * kBlockBytes, &tm_k, 64 * blk, y,
-                               &bar[C::kKFull + s]);
+                    copy_tile(sK + s * C::kTile, &tm_k, j, &bar[C::kKFull + s]);
                     ++gk;
-                    if (pend_y >= 0 && !issue_v(pend_y)) {
+                    if (pend >= 0 && !issue_v(pend)) {
                         stop = true;
                         break;
                     }
-                    pend_y = y;
+                    pend = j;
                 }
                 // the item's last value tile now, not behind the next item's
                 // query-buffer wait (its P V would stall on the load)
-                if (!stop && pend_y >= 0) stop = !issue_v(pend_y);
-                pend_y = -1;
+                if (!stop && pend >= 0) stop = !issue_v(pend);
+                pend = -1;
             }
             // let every copy issued land before the CTA may exit
-            for (int x = 0; x < kSlots; x++)
-                if (uq[x] > 0)
-                    mbar_wait_bounded(&bar[C::kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
-            for (int64_t x = gk - C::kKStages; x < gk; x++)
-                if (x >= 0)
-                    mbar_wait_bounded(&bar[C::kKFull + (int)(x % C::kKStages)], (uint32_t)((x / C::kKStages) & 1),
-                                      err);
-            for (int64_t x = gv - C::kVStages; x < gv; x++)
-                if (x >= 0)
-                    mbar_wait_bounded(&bar[C::kVFull + (int)(x % C::kVStages)], (uint32_t)((x / C::kVStages) & 1),
-                                      err);
+            if (lane == 0) {
+                for (int x = 0; x < kSlots; x++)
+                    if (uq[x] > 0)
+                        mbar_wait_bounded(&bar[C::kQFull + x], (uint32_t)((uq[x] - 1) & 1), err);
+                for (int64_t x = gk - C::kKStages; x < gk; x++)
+                    if (x >= 0)
+                        mbar_wait_bounded(&bar[C::kKFull + (int)(x % C::kKStages)],
+                                          (uint32_t)((x / C::kKStages) & 1), err);
+                for (int64_t x = gv - C::kVStages; x < gv; x++)
+                    if (x >= 0)
+                        mbar_wait_bounded(&bar[C::kVFull + (int)(x % C::kVStages)],
+                                          (uint32_t)((x / C::kVStages) & 1), err);
+            }
         }
     } else if (warp == 1) {
         // ===================== MMA issue =====================
@@ -733,29 +854,38 @@ cudaError_t launch_prefill_d(const PrefillArgs &a, int num_sms, cudaStream_t str
         const cuuint32_t box[3] = {64, 1, kBM};
         if (!encode(&tq, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
     }
+    const bool paged = a.map.table != nullptr;
     {
-        const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)(a.cache_rows * a.H_kv)};
+        // the cache rows as one 2-D array: contiguous caches cache_rows x
+        // H_kv rows, tiles of 128 rows; pages num_blocks x H_kv x block_size
+        // rows, one box per page (at most 128 rows)
+        const int64_t bs = (int64_t)1 << a.map.bs_log2;
+        const cuuint64_t rows = paged ? (cuuint64_t)(a.map.num_blocks * a.H_kv * bs)
+                                      : (cuuint64_t)(a.cache_rows * a.H_kv);
+        const cuuint64_t dims[2] = {(cuuint64_t)D, rows};
         const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-        const cuuint32_t box[2] = {64, kBN};
+        const cuuint32_t box[2] = {64, (cuuint32_t)(paged && bs < kBN ? bs : kBN)};
         if (!encode(&tk, a.k_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
         if (!encode(&tv, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
     }
-    auto kern = prefill_attn_kernel<D>;
+    auto kern = paged ? prefill_attn_kernel<D, true> : prefill_attn_kernel<D, false>;
     // the shared-memory opt-in is per device: set it once on each
     static int configured_device_mask = 0;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (!(dev < 31 && (__atomic_load_n(&configured_device_mask, __ATOMIC_ACQUIRE) & (1 << dev)))) {
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)C::kSmemBytes);
-        if (e != cudaSuccess) return e;
+        for (auto kk : {prefill_attn_kernel<D, false>, prefill_attn_kernel<D, true>}) {
+            e = cudaFuncSetAttribute(kk, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)C::kSmemBytes);
+            if (e != cudaSuccess) return e;
+        }
         if (dev < 31) __atomic_fetch_or(&configured_device_mask, 1 << dev, __ATOMIC_ACQ_REL);
     }
     const float sl2 = a.scale * 1.4426950408889634f;
     kern<<<num_sms, kThreads, C::kSmemBytes, stream>>>(
         tq, tk, tv, a.q_off, a.P, a.T, a.N, a.cache_off, static_cast<__nv_bfloat16 *>(a.out),
-        a.q_rows, a.cache_rows, sl2, a.B, a.H_q, a.H_kv, a.w_eff, a.err);
+        a.q_rows, a.cache_rows, sl2, a.B, a.H_q, a.H_kv, a.w_eff, a.err, a.map);
     return cudaGetLastError();
 }
 

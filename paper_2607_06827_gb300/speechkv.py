@@ -60,6 +60,9 @@ SIGNATURES = {
     "speechkv_prefill_attn": (ctypes.c_int, [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _I64, _P, _F,
                                              _I32, _I32, _I32, _I32, _I32, _I32, _I32,
                                              ctypes.c_int, _P]),
+    "speechkv_prefill_attn_paged": (ctypes.c_int, [_P, _P, _I64, _P, _P, _P, _P, _P, _P, _I32,
+                                                   _I32, _I64, _P, _F, _I32, _I32, _I32, _I32,
+                                                   _I32, _I32, _I32, ctypes.c_int, _P]),
     "speechkv_check_device_error": (ctypes.c_int, [_P]),
     "speechkv_selftest_timeout": (ctypes.c_int, [_P]),
 }
@@ -285,6 +288,21 @@ def prefill_attn(q, q_off, P, T, N, k_cache, v_cache, cache_off, out, w: int, la
         _ptr(cache_off), cache_rows, _ptr(out), float(scale), B, H_q, H_kv, d, w, layer, l0,
         _dtype_code(q), _stream(stream)),
         "speechkv_prefill_attn")
+
+
+def prefill_attn_paged(q, q_off, P, T, N, k_pages, v_pages, block_table, out, w: int,
+                       layer: int, l0: int, scale: float = 0.0, stream=None):
+    """speechkv_prefill_attn_paged: as prefill_attn(), over pages
+    [num_blocks, H_kv, block_size, d] through block_table [B, max_blocks]."""
+    q_rows, H_q, d = q.shape
+    B = P.numel()
+    H_kv = k_pages.shape[1]
+    nb, bs = _pages(k_pages, block_table)
+    _check(load().speechkv_prefill_attn_paged(
+        _ptr(q), _ptr(q_off), q_rows, _ptr(P), _ptr(T), _ptr(N), _ptr(k_pages), _ptr(v_pages),
+        _ptr(block_table), block_table.shape[1], bs, nb, _ptr(out), float(scale), B, H_q, H_kv,
+        d, w, layer, l0, _dtype_code(q), _stream(stream)),
+        "speechkv_prefill_attn_paged")
 
 
 def check_device_error(stream=None) -> int:

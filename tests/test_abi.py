@@ -1,6 +1,7 @@
 """The C-ABI library builds for sm_103a, loads, and exports every entry point
 include/speechkv.h declares; host-only helpers and host-side argument checks
 work without a GPU (no kernel is launched here)."""
+import ctypes
 import os
 import re
 
@@ -109,6 +110,15 @@ def test_host_argument_checks_without_gpu():
     assert lib.speechkv_prefill_attn(*pf(1, 10, 1 << 28, 16, 8, 128, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_prefill_attn(*pf(0, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.OK
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
+    # paged prefill: pages of at least 8 rows; table required
+    fake = ctypes.c_void_p(256)  # never dereferenced: every call below fails a host check
+    pfp = lambda B, tab, bs, d: (  # noqa: E731
+        z, z, 10, z, z, z, z, z, tab, 4, bs, 8, z, 0.0, B, 16, 8, d, 4, 0, 0, sk.BF16, z)
+    assert lib.speechkv_prefill_attn_paged(*pfp(0, z, 16, 128)) == sk.OK
+    assert lib.speechkv_prefill_attn_paged(*pfp(1, z, 16, 128)) == sk.ERR_INVALID_ARG   # no table
+    assert lib.speechkv_prefill_attn_paged(*pfp(1, fake, 4, 128)) == sk.ERR_UNSUPPORTED  # 4-row pages
+    assert lib.speechkv_prefill_attn_paged(*pfp(1, fake, 16, 96)) == sk.ERR_UNSUPPORTED
+    assert lib.speechkv_prefill_attn_paged(*pfp(1, fake, 16, 128)) == sk.ERR_INVALID_ARG  # NULLs
 
 
 def test_workspace_size_explicit_grid():

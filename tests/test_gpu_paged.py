@@ -1,9 +1,12 @@
 """GPU tests of the paged cache layout (block tables, as in the paper's
-serving system): speechkv_pool_paged, speechkv_append_paged and
-speechkv_decode_step_paged against the contiguous entry points on the same
-inputs.  Paging only moves rows, and the paged path splits the work the same
-way, so caches, lengths and outputs must be bit-identical; one case is also
-checked against the oracle directly."""
+serving system): speechkv_pool_paged, speechkv_append_paged,
+speechkv_decode_step_paged and speechkv_prefill_attn_paged against the
+contiguous entry points on the same inputs.
+Paging only moves rows: caches and lengths must be bit-identical, and so
+must the fp32 decode outputs and the prefill outputs; bf16 decode outputs
+are equal up to summation order (over a block table the decode tiles start
+on 16-row boundaries).  One case is also checked against the oracle
+directly."""
 import dataclasses
 
 import numpy as np
@@ -167,3 +170,52 @@ def test_paged_invalid_block_is_reported():
         assert int(tb[b, n // 64]) in changed
     assert all(int(x) in {int(tb[1, int(L.len[1]) // 64]), int(tb[2, int(L.len[2]) // 64])}
                for x in changed)
+
+
+def _prefill_q(wl, layer):
+    qs = [inputs.prefill_q(wl, layer, b) for b in range(wl.B)]
+    q_off = torch.from_numpy(np.concatenate([[0], np.cumsum(wl.full_rows())]).astype(np.int64))
+    return torch.cat(qs).cuda(), q_off.cuda()
+
+
+@pytest.mark.parametrize("block_size,layer", [(8, 8), (16, 8), (64, 8), (128, 8), (256, 8),
+                                              (16, 0), (128, 0)])
+def test_paged_prefill_matches_contiguous(block_size, layer):
+    """speechkv_prefill_attn_paged over the pages speechkv_pool_paged wrote:
+    bit-identical to speechkv_prefill_attn over the contiguous cache (a
+    pooled layer and a full-resolution one; pages smaller than, equal to and
+    larger than a 128-row key tile)."""
+    sk = H.lib()
+    wl = inputs.qwen_ragged(B=4)
+    wl = dataclasses.replace(wl, G=[0] * wl.B)  # the prompt only (before any decoding)
+    L, pg, _ = _prefill_both(wl, layer, 0, block_size, seed=block_size + layer)
+    _same_cache(wl, L, pg)
+    q, q_off = _prefill_q(wl, layer)
+    P, T, N = H.lengths_dev(wl)
+    o1, o2 = torch.full_like(q, 7.0), torch.full_like(q, 5.0)
+    sk.prefill_attn(q, q_off, P, T, N, L.k, L.v, L.cache_off, o1, wl.w, layer, wl.l0, wl.H_kv)
+    sk.prefill_attn_paged(q, q_off, P, T, N, pg.k, pg.v, pg.table, o2, wl.w, layer, wl.l0)
+    assert sk.check_device_error() == sk.OK
+    assert torch.equal(o1, o2)
+
+
+def test_paged_prefill_invalid_block_is_reported():
+    """A block-table entry of -1 inside a request's rows: the paged prefill
+    reports an invalid argument (the rows are read from page 0 instead, no
+    fault); the other requests' outputs are unaffected."""
+    sk = H.lib()
+    wl = inputs.qwen_ragged(B=3)
+    wl = dataclasses.replace(wl, G=[0] * wl.B)
+    layer = wl.l0
+    L, pg, _ = _prefill_both(wl, layer, 0, 16, seed=12)
+    table = pg.table.clone()
+    table[0, 1] = -1
+    q, q_off = _prefill_q(wl, layer)
+    P, T, N = H.lengths_dev(wl)
+    o1, o2 = torch.zeros_like(q), torch.zeros_like(q)
+    sk.prefill_attn(q, q_off, P, T, N, L.k, L.v, L.cache_off, o1, wl.w, layer, wl.l0, wl.H_kv)
+    assert sk.check_device_error() == sk.OK
+    sk.prefill_attn_paged(q, q_off, P, T, N, pg.k, pg.v, table, o2, wl.w, layer, wl.l0)
+    assert sk.check_device_error() == sk.ERR_INVALID_ARG
+    off = q_off.cpu().numpy()
+    assert torch.equal(o1[off[1]:], o2[off[1]:])
