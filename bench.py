@@ -1212,6 +1212,8 @@ def main():
                 "step_gbs": round(r["step_gbs"], 1),
                 "attn_us_compressed_layer": round(r["attn_us_compressed_layer"], 2),
                 "attn_gbs_compressed_layer": round(r["attn_gbs_compressed_layer"], 1),
+                "frac_compressed_layer": round(r["attn_gbs_compressed_layer"] /
+                                               measured_peak()[0], 4),
                 "w1_us_per_step_per_layer": round(w1["us_per_step_per_layer"], 2) if w1 else None,
                 "w1_attn_us_same_layer": round(w1["attn_us_compressed_layer"], 2) if w1 else None,
                 "speedup_vs_w1_compressed_layer": (round(w1["attn_us_compressed_layer"] /

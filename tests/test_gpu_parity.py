@@ -512,16 +512,18 @@ def test_full_size_long_audio_fused(sk, oracle):
     _sampled_full_size(sk, oracle, wl, wl.l0, samples=[3], fused=True)
 
 
-def test_max_batch_fused_step(sk, oracle):
+@pytest.mark.parametrize("H_q,H_kv", [(16, 8), (32, 4)])
+def test_max_batch_fused_step(sk, oracle, H_q, H_kv):
     """B = SPEECHKV_MAX_BATCH (the largest per-request tables in shared
     memory), short random lengths: pooling, one fused decode step, sampled
-    requests against the oracle."""
+    requests against the oracle (2 and 8 query heads per KV head: the
+    8-head instance has the largest merge buffers)."""
     rng = np.random.default_rng(4242)
     B = sk.MAX_BATCH
     T = [int(x) for x in rng.integers(1, 60, B)]
     N = [int(x) for x in rng.integers(0, 20, B)]
-    wl = inputs.Workload(name="maxbatch", dtype="bf16", L=28, l0=8, w=4, H_q=16, H_kv=8, d=128,
-                         P=[0] * B, T=T, N=N, G=[0] * B, steps=1, seed=4242)
+    wl = inputs.Workload(name="maxbatch", dtype="bf16", L=28, l0=8, w=4, H_q=H_q, H_kv=H_kv,
+                         d=128, P=[0] * B, T=T, N=N, G=[0] * B, steps=1, seed=4242)
     layer = wl.l0
     L, (ks, vs, gate) = H.gpu_prefill(wl, layer, extra_rows=1)
     ws = sk.new_workspace(wl.B, wl.H_q, wl.H_kv, wl.d)
