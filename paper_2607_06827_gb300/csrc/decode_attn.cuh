@@ -174,7 +174,7 @@ struct Partition {
 // CTAs used for U units on a grid of `grid`: at least kMinUnitsPerCta units
 // each (a small batch spread over every SM would only multiply the partial
 // results each (request, head) has to merge), at most the grid.
-constexpr int64_t kMinUnitsPerCta = 64;
+constexpr int64_t kMinUnitsPerCta = 256;
 __device__ __forceinline__ int64_t ctas_for(int64_t U, int64_t grid) {
     const int64_t n = (U + kMinUnitsPerCta - 1) / kMinUnitsPerCta;
     return n < grid ? n : grid;
