@@ -184,7 +184,7 @@ __device__ __forceinline__ int64_t ctas_for(int64_t U, int64_t grid) {
 // previous kernel (programmatic dependent launch with
 // SPEECHKV_OVERLAP_PRIOR).
 #ifndef SPEECHKV_PRE_WAIT_TILES
-#define SPEECHKV_PRE_WAIT_TILES 3
+#define SPEECHKV_PRE_WAIT_TILES 2
 #endif
 constexpr int kPreWaitTiles = SPEECHKV_PRE_WAIT_TILES;
 
