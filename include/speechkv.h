@@ -387,7 +387,7 @@ speechkv_status speechkv_decode_step_noalloc(
  *              decode step reads a tile in 16-row groups aligned to the
  *              rows' index (bf16: one copy per group and page, issued in
  *              parallel): measured against the contiguous layout, 64-row
- *              pages cost 4-7 %, 16-row pages (vLLM's default) 7-13 %.
+ *              pages cost 4-7 %, 16-row pages (vLLM's default) 7-14 %.
  * num_blocks   host: pages in k_pages / v_pages (bounds the table entries).
  * The other arguments, the results and the errors are those of the
  * contiguous entry point of the same name (the rows and their order are the
