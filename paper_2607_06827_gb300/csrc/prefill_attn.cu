@@ -16,7 +16,9 @@
 //   * warp 0 lane 0: TMA tensor copies (128-byte swizzle) of the two query
 //     tiles and of 128-row key tiles (three stages) and value tiles (two
 //     stages), keys one tile ahead of values;
-//   * warp 1 lane 0: tcgen05.mma issue -- per key tile and slot x,
+//   * warp 1: tcgen05.mma issue, the warp converged and one elected lane
+//     issuing (a lone issuing thread was slowed more by the softmax warps'
+//     instruction issue on its sub-partition) -- per key tile and slot x,
 //     O_x += P_x V then S_x = Q_x K^T of the next key tile, into 128-column
 //     TMEM buffers (S_0, S_1, O_0, O_1: all 512 columns); P_x is stored over
 //     the first half of S_x and read as the A operand from TMEM, so a slot's
@@ -157,11 +159,14 @@ __device__ __forceinline__ uint32_t instr_desc(bool b_mn_major, int n) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
            ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kBM >> 4) << 24);
 }
+// tcgen05.mma (A and B in shared memory), issued by one elected lane of a
+// converged warp: the whole warp runs the issue loop, so the descriptors and
+// counters are warp-uniform values.
 __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t id,
                                      uint32_t accumulate) {
     asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "{\n\t.reg .pred p, e;\n\telect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
         "l"(a), "l"(b), "r"(id), "r"(accumulate));
 }
 // The same with the A operand in TMEM: row m in lane m, two bf16 per 32-bit
@@ -169,15 +174,16 @@ __device__ __forceinline__ void umma(uint32_t d_tmem, uint64_t a, uint64_t b, ui
 __device__ __forceinline__ void umma_tmem_a(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
                                             uint32_t id, uint32_t accumulate) {
     asm volatile(
-        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "{\n\t.reg .pred p, e;\n\telect.sync _|e, 0xffffffff;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "@e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
         "r"(a_tmem), "l"(b), "r"(id), "r"(accumulate));
 }
-// Arrive on `bar` once every tcgen05 operation issued so far by this thread
-// has completed.
+// Arrive on `bar` (one elected lane) once every tcgen05 operation issued so
+// far by this warp has completed.
 __device__ __forceinline__ void umma_commit(uint64_t *bar) {
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+        "{\n\t.reg .pred e;\n\telect.sync _|e, 0xffffffff;\n\t"
+        "@e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n\t}" ::"r"(
             smem_addr(bar))
         : "memory");
 }
@@ -577,8 +583,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         // P_x lives in the first half of S_x's columns, so slot x's next
         // Q K^T waits for its P V to complete; the other slot's products keep
         // the tensor pipe busy meanwhile, and each slot's softmax overlaps
-        // the other slot's products.
-        if (lane == 0) {
+        // the other slot's products.  The whole warp runs this loop (its
+        // waits agree through a vote) and one elected lane issues.
+        {
+            auto wb = [&](uint64_t *bb, uint32_t par) -> bool {
+                return __all_sync(0xffffffffu, wait_bar(bb, par, abort, err));
+            };
             const uint32_t id_qk = instr_desc(false, kBN), id_pv = instr_desc(true, D);
             const uint32_t aQ = smem_addr(sQ), aK = smem_addr(sK), aV = smem_addr(sV);
             // Descriptors are built once per buffer; a K step or a stage only
@@ -592,10 +602,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool issued = false, stop = false;
             auto qk = [&](int x, int64_t gg) -> bool {  // S_x = Q_x K^T of key tile gg
                 const int s = (int)(gg % C::kKStages);
-                if (x == 0 && !wait_bar(&bar[C::kKFull + s], (uint32_t)((gg / C::kKStages) & 1), abort, err))
+                if (x == 0 && !wb(&bar[C::kKFull + s], (uint32_t)((gg / C::kKStages) & 1)))
                     return false;
                 // P V of slot x's previous tile has read P_x (inside S_x)
-                if (ut[x] > 0 && !wait_bar(&bar[C::kODone + x], (uint32_t)((ut[x] - 1) & 1), abort, err))
+                if (ut[x] > 0 && !wb(&bar[C::kODone + x], (uint32_t)((ut[x] - 1) & 1)))
                     return false;
                 tc_fence_after();
                 const uint64_t dQx = dQ + (uint64_t)x * kStageD, dKs = dK + (uint64_t)s * kStageD;
@@ -608,7 +618,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 issued = true;
                 return true;
             };
-            for (int64_t k = blockIdx.x; k < total && !stop && !*abort; k += gridDim.x) {
+            for (int64_t k = blockIdx.x;
+                 k < total && !stop && !__shfl_sync(0xffffffffu, (int)*abort, 0); k += gridDim.x) {
                 Req q;
                 const Item item = item_at(k, tiles_max, H_q, H_kv, tab, q);
                 if (!item.valid) continue;
@@ -617,7 +628,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int64_t tl = min(t0 + kBM, (int64_t)q.S) - 1;
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
                 for (int x = 0; x < n && !stop; x++)
-                    stop = !wait_bar(&bar[C::kQFull + x], (uint32_t)(uq[x] & 1), abort, err);
+                    stop = !wb(&bar[C::kQFull + x], (uint32_t)(uq[x] & 1));
                 for (int x = 0; x < n && !stop; x++) stop = !qk(x, g);
                 if (stop) break;
                 umma_commit(&bar[C::kKEmpty + (int)(g % C::kKStages)]);
@@ -626,9 +637,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int j = 0; j < n_kt && !stop; j++, g++) {
                     const int sv = (int)(g % C::kVStages);
                     for (int x = 0; x < n; x++) {
-                        if (!wait_bar(&bar[C::kPFull + x], (uint32_t)(ut[x] & 1), abort, err) ||
+                        if (!wb(&bar[C::kPFull + x], (uint32_t)(ut[x] & 1)) ||
                             (x == 0 &&
-                             !wait_bar(&bar[C::kVFull + sv], (uint32_t)((g / C::kVStages) & 1), abort, err))) {
+                             !wb(&bar[C::kVFull + sv], (uint32_t)((g / C::kVStages) & 1)))) {
                             stop = true;
                             break;
                         }
