@@ -469,14 +469,16 @@ __global__ void __launch_bounds__(kThreads, 1)
             // for the stages, sets the expected bytes and copies the queries,
             // and lane p copies page p of a key or value tile (pages of 8
             // rows or more: at most 16 per 128-row tile), so that the small
-            // copies are issued in parallel.  Pages past the compressed rows
-            // are not read (their rows are masked, and the values zeroed, by
-            // the softmax warps).
+            // copies are issued in parallel.  Each lane reads its block-table
+            // entry one key tile ahead of the copies that need it (a cold
+            // entry read in front of every tile's copies set the producer's
+            // pace).  Pages past the compressed rows are not read (their rows
+            // are masked, and the values zeroed, by the softmax warps).
             int64_t uq[kSlots] = {}, gk = 0, gv = 0;  // query (per slot), key, value tiles issued
-            int pend = -1;                            // key tile whose values are still to issue
             bool stop = false;
             const int lg = map.bs_log2;
-            const int rows = lg < 7 ? 1 << lg : kBN;  // rows per copy (the maps' box)
+            const int lgr = lg < 7 ? lg : 7;  // rows per copy (the maps' box): 1 << lgr
+            const int rows = 1 << lgr;
             auto wait0 = [&](uint64_t *b, uint32_t parity) -> bool {  // lane 0 waits for all
                 int ok = 1;
                 if (lane == 0) ok = wait_bar(b, parity, abort, err);
@@ -492,17 +494,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int n_kt = (int)(pi_of(q, tl, w) / kBN) + 1;
                 const int hk = item.hq0 / G;                      // the KV head
                 const int64_t crows = (int64_t)q.P + q.n + q.N;  // compressed rows
-                auto copy_tile = [&](unsigned char *dst, const CUtensorMap *tm, int kt,
+                const int32_t *row_table = map.table + (int64_t)item.b * map.max_blocks;
+                // Lane p's page of key tile kt (its copies are issued only
+                // where ncopy(kt) > p); read one tile ahead of its copies.
+                auto entry = [&](int kt) -> int32_t {
+                    const int64_t r = (int64_t)kt * kBN + ((int64_t)lane << lgr);
+                    return kt < n_kt && r < crows ? __ldg(row_table + (r >> lg)) : 0;
+                };
+                auto ncopy_of = [&](int kt) -> int {  // segments of tile kt that hold rows
+                    const int64_t left = crows - (int64_t)kt * kBN;
+                    if (left <= 0) return 0;
+                    const int64_t c = (left + rows - 1) >> lgr;
+                    return c < kBN / rows ? (int)c : kBN / rows;
+                };
+                auto copy_tile = [&](unsigned char *dst, const CUtensorMap *tm, int kt, int32_t blk_id,
                                      uint64_t *fb) {
-                    const int64_t r0 = (int64_t)kt * kBN;
-                    int ncopy = 0;
-                    while (ncopy < kBN / rows && r0 + (int64_t)ncopy * rows < crows) ncopy++;
+                    const int ncopy = ncopy_of(kt);
                     if (lane == 0) mbar_arrive_expect_tx(fb, (uint32_t)(ncopy * rows * 128 * C::kBlocks));
                     __syncwarp();
                     if (lane < ncopy) {
-                        const int64_t r = r0 + (int64_t)lane * rows;
-                        int32_t blk_id =
-                            __ldg(map.table + (int64_t)item.b * map.max_blocks + (r >> lg));
+                        const int64_t r = (int64_t)kt * kBN + ((int64_t)lane << lgr);
                         if (blk_id < 0 || blk_id >= map.num_blocks) {
                             report_error(err, SPEECHKV_ERR_INVALID_ARG);  // read page 0 instead
                             blk_id = 0;
@@ -515,12 +526,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                    fb);
                     }
                 };
-                auto issue_v = [&](int kt) -> bool {
+                auto issue_v = [&](int kt, int32_t blk_id) -> bool {
                     const int s = (int)(gv % C::kVStages);
                     const int64_t u = gv / C::kVStages;
                     if (gv >= C::kVStages && !wait0(&bar[C::kVEmpty + s], (uint32_t)((u - 1) & 1)))
                         return false;
-                    copy_tile(sV + s * C::kTile, &tm_v, kt, &bar[C::kVFull + s]);
+                    copy_tile(sV + s * C::kTile, &tm_v, kt, blk_id, &bar[C::kVFull + s]);
                     ++gv;
                     return true;
                 };
@@ -540,7 +551,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     ++uq[x];
                 }
+                int32_t e_cur = entry(0), e_prev = 0;  // this lane's page of tiles j and j - 1
                 for (int j = 0; j < n_kt && !stop; j++) {
+                    const int32_t e_next = entry(j + 1);  // in flight during this tile's waits
                     // keys are free once their Q K^T is done, values once their P V is
                     const int s = (int)(gk % C::kKStages);
                     const int64_t u = gk / C::kKStages;
@@ -548,18 +561,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                         stop = true;
                         break;
                     }
-                    copy_tile(sK + s * C::kTile, &tm_k, j, &bar[C::kKFull + s]);
+                    copy_tile(sK + s * C::kTile, &tm_k, j, e_cur, &bar[C::kKFull + s]);
                     ++gk;
-                    if (pend >= 0 && !issue_v(pend)) {
+                    if (j > 0 && !issue_v(j - 1, e_prev)) {
                         stop = true;
                         break;
                     }
-                    pend = j;
+                    e_prev = e_cur;
+                    e_cur = e_next;
                 }
                 // the item's last value tile now, not behind the next item's
                 // query-buffer wait (its P V would stall on the load)
-                if (!stop && pend >= 0) stop = !issue_v(pend);
-                pend = -1;
+                if (!stop) stop = !issue_v(n_kt - 1, e_prev);
             }
             // let every copy issued land before the CTA may exit
             if (lane == 0) {
