@@ -430,7 +430,8 @@ speechkv_status speechkv_decode_step_paged(
  * (a key tile is copied as one piece per page of whole 8-row swizzle atoms;
  * SPEECHKV_ERR_UNSUPPORTED below that); num_blocks * H_kv * block_size must
  * stay below 2^31.  Pages past a request's compressed rows are not read.
- * Results are bit-identical to speechkv_prefill_attn over the same rows.
+ * Results are bit-identical to speechkv_prefill_attn over the same rows;
+ * measured against it, 16-row pages cost 2-3 %.
  */
 speechkv_status speechkv_prefill_attn_paged(
     const void *q, const int64_t *q_off, int64_t q_rows, const int32_t *P,
