@@ -46,7 +46,10 @@ def _load():
     with _lock:
         if _lib is not None:
             return _lib
-        lib = ctypes.CDLL(build())
+        # SPEECHKV_ORACLE_LIB names another build of this file's C source;
+        # only the planted-mistake test sets it, to run the pins against a
+        # copy of the oracle with one deliberate error.
+        lib = ctypes.CDLL(os.environ.get("SPEECHKV_ORACLE_LIB") or build())
         lib.oracle_round_bf16.restype = ctypes.c_double
         lib.oracle_round_bf16.argtypes = [ctypes.c_double]
         lib.oracle_round_f32.restype = ctypes.c_double

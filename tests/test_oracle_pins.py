@@ -27,6 +27,17 @@ def _rand(seed, *shape):
     return np.random.default_rng(seed).standard_normal(shape)
 
 
+def _to_storage(x, storage):
+    """Library rounding of exact values to a storage type: numpy's float32
+    conversion (IEEE round to nearest even); torch's bf16 of that fp32 value
+    (equal to bf16 of the exact value except at double-rounding ties, which
+    random data does not hit)."""
+    f32 = np.asarray(x, dtype=np.float64).astype(np.float32)
+    if storage == 1:
+        return f32.astype(np.float64)
+    return torch.from_numpy(f32).to(torch.bfloat16).double().numpy()
+
+
 def _read_golden(name):
     rows = []
     with open(os.path.join(GOLDEN, name)) as f:
@@ -235,6 +246,22 @@ def test_pool_storage_rounding(oracle):
     assert np.abs(Kb - Ke).max() <= 2**-8 * np.abs(Ke).max()
 
 
+def test_pool_text_rows_rounded_once(oracle):
+    """Text rows (before and after the speech) are copied and rounded once to
+    the storage type, like every other value the pooling produces."""
+    P, T, N, H, d, w = 3, 8, 2, 2, 8, 4
+    K, V = _rand(23, P + T + N, H, d), _rand(24, P + T + N, H, d)
+    u = _rand(25, H, d)
+    n = -(-T // w)
+    for storage in (oracle.STORE_F32, oracle.STORE_BF16):
+        Ko, Vo = oracle.pool_request(K, V, P, T, N, u, w, 0, 0, storage=storage)
+        for src, out in ((K, Ko), (V, Vo)):
+            text_in = np.concatenate([src[:P], src[P + T:]])
+            text_out = np.concatenate([out[:P], out[P + n:]])
+            assert not np.array_equal(text_out, text_in)
+            np.testing.assert_array_equal(text_out, _to_storage(text_in, storage))
+
+
 # --------------------------------------------------------------------------
 # append
 # --------------------------------------------------------------------------
@@ -343,6 +370,17 @@ def test_attn_extreme_logits(oracle):
         for hq in range(H_q):
             best = int(np.argmax(Ks[:, 0] @ q[hq]))
             np.testing.assert_allclose(out[hq], Vs[best, 0], atol=1e-12)
+
+
+def test_attn_output_rounded_once(oracle):
+    """The attention output is the exact result rounded once to storage."""
+    H_q, H_kv, d, n = 4, 2, 16, 33
+    q, K, V = _rand(44, H_q, d), _rand(45, n, H_kv, d), _rand(46, n, H_kv, d)
+    exact = oracle.decode_attn_request(q, K, V)
+    for storage in (oracle.STORE_F32, oracle.STORE_BF16):
+        out = oracle.decode_attn_request(q, K, V, storage=storage)
+        assert not np.array_equal(out, exact)
+        np.testing.assert_array_equal(out, _to_storage(exact, storage))
 
 
 # --------------------------------------------------------------------------
@@ -460,6 +498,18 @@ def test_prefill_equal_keys_average_visible_values(oracle):
         for hq in range(H_q):
             ref = V[mask[t], hq // 2].mean(axis=0)
             np.testing.assert_allclose(out[t, hq], ref, rtol=0, atol=1e-12)
+
+
+def test_prefill_output_rounded_once(oracle):
+    """Each prefill output row is the exact result rounded once to storage."""
+    P, T, N, w, H_q, H_kv, d = 2, 11, 3, 4, 4, 2, 16
+    c = len(_first_source(P, T, N, w))
+    Q, K, V = _rand(102, P + T + N, H_q, d), _rand(103, c, H_kv, d), _rand(104, c, H_kv, d)
+    exact = oracle.prefill_attn_request(Q, K, V, P, T, N, w)
+    for storage in (oracle.STORE_F32, oracle.STORE_BF16):
+        out = oracle.prefill_attn_request(Q, K, V, P, T, N, w, storage=storage)
+        assert not np.array_equal(out, exact)
+        np.testing.assert_array_equal(out, _to_storage(exact, storage))
 
 
 def test_prefill_brute_force_tiny_case(oracle):
