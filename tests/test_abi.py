@@ -98,7 +98,7 @@ def test_host_argument_checks_without_gpu():
     dp = lambda B: (*([z] * 6), 4, 48, 8, z, z, 0.0, B, 16, 8, 128, 4, 0, 0, 0, z, 0, sk.BF16, 0, z)  # noqa: E731
     assert lib.speechkv_decode_step_paged(*dp(0)) == sk.OK
     assert lib.speechkv_decode_step_paged(*dp(1)) == sk.ERR_INVALID_ARG          # no table
-    # prefill attention: bf16 and d = 128 only; 32-bit tensor-copy coordinates
+    # prefill attention: bf16 and d = 64 or 128 only; 32-bit tensor-copy coordinates
     pf = lambda B, q_rows, cache_rows, H_q, H_kv, d, w, dt: (  # noqa: E731
         z, z, q_rows, z, z, z, z, z, z, cache_rows, z, 0.0, B, H_q, H_kv, d, w, 0, 0, dt, z)
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.F32)) == sk.ERR_UNSUPPORTED
@@ -110,6 +110,7 @@ def test_host_argument_checks_without_gpu():
     assert lib.speechkv_prefill_attn(*pf(1, 10, 1 << 28, 16, 8, 128, 4, sk.BF16)) == sk.ERR_UNSUPPORTED
     assert lib.speechkv_prefill_attn(*pf(0, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.OK
     assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 128, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
+    assert lib.speechkv_prefill_attn(*pf(1, 10, 10, 16, 8, 64, 4, sk.BF16)) == sk.ERR_INVALID_ARG  # NULLs
     # paged prefill: pages of at least 8 rows; table required
     fake = ctypes.c_void_p(256)  # never dereferenced: every call below fails a host check
     pfp = lambda B, tab, bs, d: (  # noqa: E731
