@@ -36,6 +36,49 @@ def test_library_exports_every_declared_symbol():
     assert set(sk.SIGNATURES) == set(_declared())
 
 
+_C_TO_CTYPES = {
+    "int32_t": ctypes.c_int32, "int64_t": ctypes.c_int64, "uint32_t": ctypes.c_uint32,
+    "size_t": ctypes.c_size_t, "float": ctypes.c_float, "speechkv_status": ctypes.c_int,
+    "speechkv_dtype": ctypes.c_int, "cudaStream_t": ctypes.c_void_p,
+}
+
+
+def _ctype_of(decl: str):
+    """ctypes class of a C parameter or return type from the header."""
+    decl = " ".join(decl.replace("const ", "").split())
+    if "*" in decl:
+        return ctypes.c_char_p if decl.startswith("char") else ctypes.c_void_p
+    base = decl.split()[0]
+    return _C_TO_CTYPES[base]
+
+
+def _prototypes():
+    src = re.sub(r"/\*.*?\*/", "", open(HEADER).read(), flags=re.S)
+    protos = {}
+    for m in re.finditer(r"([A-Za-z_][\w \t\*]*?)\b(speechkv_[a-z_]+)\s*\(([^)]*)\)\s*;", src):
+        params = [a.strip() for a in m.group(3).split(",") if a.strip() and a.strip() != "void"]
+        # drop the parameter name (the last identifier), keep the type
+        types = [re.sub(r"\b\w+$", "", a).strip() for a in params]
+        protos[m.group(2)] = (m.group(1).strip(), types)
+    return protos
+
+
+def test_binding_signatures_match_header():
+    """Every ctypes signature of the binding has the header's argument count
+    and, position by position, the same kind of value (pointer, 32- or
+    64-bit integer, size_t, float, enum); a mismatch would pass wrong values
+    across the boundary without any error."""
+    sk = H.lib()
+    protos = _prototypes()
+    assert set(protos) == set(sk.SIGNATURES)
+    for name, (ret, types) in protos.items():
+        restype, argtypes = sk.SIGNATURES[name]
+        assert restype is _ctype_of(ret), f"{name}: return {ret}"
+        assert len(argtypes) == len(types), f"{name}: {len(argtypes)} args bound, {len(types)} declared"
+        for i, (got, decl) in enumerate(zip(argtypes, types)):
+            assert got is _ctype_of(decl), f"{name}: argument {i} ({decl}) bound as {got.__name__}"
+
+
 def test_compressed_len_matches_oracle(oracle):
     sk = H.lib()
     for wl in (inputs.qwen_ragged(), inputs.tiny_fp32(), inputs.qwen_single(),
