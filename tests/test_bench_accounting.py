@@ -9,9 +9,13 @@ length (speech pooled in windows of w from l0 on, Eq. (pool)).  The
 committed ncu traffic figures feed roofline.traffic only while they were
 taken on the current decode-kernel source.
 """
+import glob
 import os
+import shlex
 import sys
 import types
+
+import pytest
 
 from paper_2607_06827_gb300 import inputs
 from tests import harness as H
@@ -71,3 +75,22 @@ def test_traffic_scales_each_kind_by_its_own_ratio():
     rf = float(kv["full_dram_bytes_per_launch"]) / float(kv["full_algorithmic_bytes"])
     assert 1.0 <= rp < 1.1 and 1.0 <= rf < 1.1
     assert bench.profiled_traffic(res) == round((20 * rp * 100.0 + 8 * rf * 400.0) / 28)
+
+
+def test_profile_commands_parse(monkeypatch):
+    """Each ncu summary under profiles/ names the bench command it captured;
+    every such command must still be accepted by the bench's arguments."""
+    cmds = []
+    for path in sorted(glob.glob(os.path.join(H.ROOT, "profiles", "*"))):
+        for line in open(path):
+            line = line.strip().rstrip("\\").strip()
+            at = line.find("python bench.py")
+            if at >= 0:
+                cmds.append((os.path.basename(path), line[at + len("python bench.py"):]))
+    assert len(cmds) >= 6
+    for name, argv in cmds:
+        monkeypatch.setattr(sys, "argv", ["bench.py", *shlex.split(argv)])
+        try:
+            bench.parse_args()
+        except SystemExit:
+            pytest.fail(f"{name}: bench.py rejects {argv!r}")
